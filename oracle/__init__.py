@@ -1,0 +1,10 @@
+"""CPU oracle for the CURE repair-verify step: test infrastructure only.
+
+Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
+leg import this package; the library's product path never does.
+"""
+from .cure_oracle import (score_draft, row_argmax, select_ufps, build_tree, anc_set,
+                          cache_rows, tree_attn, accept, resync)
+
+__all__ = ["score_draft", "row_argmax", "select_ufps", "build_tree", "anc_set",
+           "cache_rows", "tree_attn", "accept", "resync"]

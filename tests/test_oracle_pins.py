@@ -1,0 +1,522 @@
+"""Pins for the CPU oracle against what the paper and mathematics fix.
+
+Nothing here re-uses the oracle's code to compute an expectation: the checks
+are hand-derived fixtures, closed forms, brute force over tiny inputs,
+textbook routines (sorting, logsumexp, scaled-dot-product attention) and
+invariants.  Each check is chosen so that a plausible mistake in the oracle
+(a dropped term, a wrong sign or index, a transposed operand, a flipped tie
+rule) fails at least one of them; ``test_pins_catch_planted_mistakes`` plants
+such mistakes in oracle outputs and confirms the checkers flag them.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_00531_gb300 import workload as W
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _num(v):
+    return float(v) if not isinstance(v, str) else float(v)
+
+
+# ---------------------------------------------------------------- S1 pins
+def test_score_hand_ties():
+    g = _load("score_ties.json")
+    for row in g["rows"]:
+        x = np.array([_num(v) for v in row["x"]], dtype=np.float64)[None, :]
+        ids, vals, margin, lse, logp1 = oracle.score_draft(x, g["k"])
+        assert ids[0].tolist() == row["ids"]
+        assert vals[0].tolist() == [_num(v) for v in row["vals"]]
+        assert margin[0] == _num(row["margin"])
+
+
+def test_lse_closed_forms():
+    # all-equal row: lse = c + ln V, logp1 = -ln V
+    for V, c in [(7, 0.0), (32000, 3.25), (151936, -11.5)]:
+        x = np.full((1, V), c)
+        _, _, m, lse, lp = oracle.score_draft(x, 2)
+        assert m[0] == 0.0
+        assert abs(lse[0] - (c + math.log(V))) < 1e-12 * max(1, abs(c) + math.log(V))
+        assert abs(lp[0] + math.log(V)) < 1e-12 * math.log(V)
+    # the hand-tie row: log(e^1 + 3 e^3 + e^2)
+    x = np.array([[1, 3, 3, 2, -np.inf, 3]], dtype=np.float64)
+    _, _, _, lse, lp = oracle.score_draft(x, 3)
+    want = math.log(math.e + 3 * math.e ** 3 + math.e ** 2)
+    assert abs(lse[0] - want) < 1e-13
+    assert abs(lp[0] - (3 - want)) < 1e-13
+    # a single finite entry: probability one
+    x = np.array([[-np.inf, 7, -np.inf, -np.inf]])
+    _, _, _, lse, lp = oracle.score_draft(x, 2)
+    assert lse[0] == 7.0 and lp[0] == 0.0
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_score_bruteforce_and_textbook(seed):
+    from scipy.special import logsumexp
+    rng = np.random.default_rng(seed)
+    V = int(rng.integers(2, 40))
+    k = int(rng.integers(1, min(8, V) + 1))
+    # few distinct values so ties are common
+    x = rng.integers(-4, 5, size=(5, V)).astype(np.float64) * 0.5
+    ids, vals, margin, lse, logp1 = oracle.score_draft(x, k)
+    for r in range(5):
+        ranked = sorted(range(V), key=lambda i: (-x[r, i], i))
+        assert ids[r].tolist() == ranked[:k]
+        assert vals[r].tolist() == [x[r, i] for i in ranked[:k]]
+        s = math.fsum(math.exp(v) for v in x[r])
+        assert abs(lse[r] - math.log(s)) < 1e-13 * max(1.0, abs(math.log(s)))
+        assert abs(lse[r] - logsumexp(x[r])) < 1e-12
+        if k >= 2:
+            # Eq. (2): the logit gap equals the log-probability gap
+            lp = x[r] - math.log(s)
+            assert abs(margin[r] - (lp[ranked[0]] - lp[ranked[1]])) < 1e-12
+        assert abs(logp1[r] - (x[r, ranked[0]] - math.log(s))) < 1e-12
+    # np.argsort(kind="stable") on the negated values is the same ranking
+    order = np.argsort(-x, axis=1, kind="stable")[:, :k]
+    assert np.array_equal(order, ids)
+
+
+def test_row_argmax_first_max():
+    x = np.array([[0, 5, 5, 1], [-1, -1, -1, -1], [3, 2, 1, 3]], dtype=np.float64)
+    assert oracle.row_argmax(x).tolist() == [1, 0, 0]
+    rng = np.random.default_rng(3)
+    x = rng.integers(0, 4, size=(50, 30)).astype(np.float64)
+    want = [min(i for i in range(30) if x[r, i] == x[r].max()) for r in range(50)]
+    assert oracle.row_argmax(x).tolist() == want
+
+
+# ---------------------------------------------------------------- S2/S3 pins
+def _tree_hand():
+    g = _load("tree_hand.json")
+    K = g["K"]
+    top = np.array(g["top_ids"])[None]
+    margin = np.array(g["margin"], dtype=np.float32)[None]
+    t = oracle.build_tree(top, margin, np.array([g["root_tok"]]), np.array([g["cache_len"]]),
+                          g["tau"], g["budget"], g["branches"], g["repair_depth"])
+    return g, t
+
+
+def test_tree_hand():
+    g, t = _tree_hand()
+    e = g["expect_tree"]
+    n = e["n_nodes"]
+    assert t["n_nodes"][0] == n
+    for key in ("tok", "parent", "depth", "pos"):
+        assert t[key][0, :n].tolist() == e[key], key
+        assert (t[key][0, n:] == -1).all()
+    assert [int(v) for v in t["anc"][0, :n, 0]] == e["anc"]
+    assert t["ufp_pos"][0].tolist() == e["ufp_pos"]
+    assert t["n_ufp"][0] == e["n_ufp"]
+
+
+def ancestors_by_parent_walk(parent_row, j):
+    s = set()
+    while j >= 0 and j not in s:          # a cycle (a corrupt tree) ends the walk
+        s.add(j)
+        j = int(parent_row[j])
+    return s
+
+
+def check_tree(t, top_ids, margin, tau, budget, branches, depth_rep, cache_len, redraft=None):
+    """Invariants of a built tree; returns a list of violations."""
+    bad = []
+    B, K, k = top_ids.shape
+    for b in range(B):
+        n = int(t["n_nodes"][b])
+        if n > 1 + K + budget:
+            bad.append(("budget", b))
+        if t["parent"][b, 0] != -1 or t["depth"][b, 0] != 0:
+            bad.append(("root", b))
+        for i in range(1, K + 1):        # branch 0 is the draft chain
+            if (t["tok"][b, i] != top_ids[b, i - 1, 0] or t["parent"][b, i] != i - 1
+                    or t["depth"][b, i] != i):
+                bad.append(("chain", b, i))
+        for j in range(n):
+            p = int(t["parent"][b, j])
+            if j > 0 and not (0 <= p < j):
+                bad.append(("parent-order", b, j))
+            if j > 0 and t["depth"][b, j] != t["depth"][b, p] + 1:
+                bad.append(("depth", b, j))
+            if t["pos"][b, j] != cache_len[b] + t["depth"][b, j]:
+                bad.append(("pos", b, j))
+            if set(oracle.anc_set(t["anc"][b, j])) != ancestors_by_parent_walk(t["parent"][b], j):
+                bad.append(("anc", b, j))
+        for j in range(n, t["tok"].shape[1]):
+            if t["tok"][b, j] != -1 or t["anc"][b, j].any():
+                bad.append(("padding", b, j))
+        # every repair node hangs under a gated position with a ranked alternative
+        repair_pos = []
+        for j in range(K + 1, n):
+            p = int(t["parent"][b, j])
+            if p <= K:                        # an alternative: child of chain node i
+                i = p
+                if not (np.float32(margin[b, i]) < np.float32(tau)):
+                    bad.append(("gate", b, j))
+                if int(t["tok"][b, j]) not in [int(v) for v in top_ids[b, i, 1:branches]]:
+                    bad.append(("alt-token", b, j))
+                repair_pos.append(i)
+            else:                             # a successor of an alternative
+                if depth_rep < 2:
+                    bad.append(("depth1-successor", b, j))
+                else:
+                    i = int(t["parent"][b, p])
+                    r = [int(v) for v in top_ids[b, i, :]].index(int(t["tok"][b, p])) + 1
+                    if t["tok"][b, j] != redraft[b, i, r - 2]:
+                        bad.append(("successor-token", b, j))
+        # ascending-margin priority: an eligible position left without any
+        # alternative never has a smaller (margin, position) than a taken one
+        # whose alternatives could have been swapped for it
+        eligible = [i for i in range(K) if np.float32(margin[b, i]) < np.float32(tau)]
+        taken = set(repair_pos)
+        for i in eligible:
+            if i in taken:
+                continue
+            cost = min(depth_rep, K - i)
+            if n - (1 + K) + cost <= budget:
+                bad.append(("fits-but-skipped", b, i))
+            for jpos in taken:
+                if (np.float32(margin[b, jpos]), jpos) > (np.float32(margin[b, i]), i) and \
+                        min(depth_rep, K - jpos) >= cost:
+                    bad.append(("priority", b, i, jpos))
+        if len(taken) != int(t["n_ufp"][b]) or set(t["ufp_pos"][b, :len(taken)].tolist()) != taken:
+            bad.append(("ufp-list", b))
+    return bad
+
+
+def _random_case(seed, K=None, budget=None, branches=None, depth_rep=1, tau=None):
+    rng = np.random.default_rng(seed)
+    B = 3
+    K = K or int(rng.integers(2, 12))
+    k = 4
+    branches = branches or int(rng.integers(2, 5))
+    budget = int(rng.integers(0, 3 * K)) if budget is None else budget
+    tau = float(rng.choice([0.0, 0.5, 1.0, 2.0])) if tau is None else tau
+    # margins on a coarse grid so that ties happen
+    margin = (rng.integers(0, 12, size=(B, K)) * 0.25).astype(np.float32)
+    top = np.stack([rng.permutation(1000)[:k] for _ in range(B * K)]).reshape(B, K, k)
+    root = rng.integers(0, 1000, size=B)
+    L = rng.integers(10, 50, size=B)
+    redraft = rng.integers(0, 1000, size=(B, K, max(1, branches - 1)))
+    return top, margin, root, L, tau, budget, branches, depth_rep, redraft
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_tree_invariants(seed):
+    depth_rep = 2 if seed % 3 == 0 else 1
+    top, margin, root, L, tau, budget, branches, d, redraft = _random_case(seed, depth_rep=depth_rep)
+    t = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft)
+    assert check_tree(t, top, margin, tau, budget, branches, d, L, redraft) == []
+
+
+def test_tree_special_cases():
+    top, margin, root, L, _, _, branches, _, redraft = _random_case(7, K=8, branches=3)
+    K = 8
+    # tau <= 0: margins are >= 0, so no position is gated: the tree is branch 0
+    t = oracle.build_tree(top, margin, root, L, 0.0, 20, branches, 1, redraft)
+    assert (t["n_nodes"] == K + 1).all() and (t["n_ufp"] == 0).all()
+    # budget 0: branch 0 only, whatever the gate says
+    t = oracle.build_tree(top, margin, root, L, 100.0, 0, branches, 1, redraft)
+    assert (t["n_nodes"] == K + 1).all()
+    # a budget that covers everything admits every gated position, every rank
+    for d in (1, 2):
+        t = oracle.build_tree(top, margin, root, L, 1.0, K * (branches - 1) * d, branches, d, redraft)
+        for b in range(3):
+            eligible = [i for i in range(K) if margin[b, i] < 1.0]
+            want = sum((branches - 1) * min(d, K - i) for i in eligible)
+            assert t["n_nodes"][b] == 1 + K + want
+    # a margin exactly at tau is not a UFP (strict gate)
+    m = np.full((1, 4), 1.0, dtype=np.float32)
+    t = oracle.build_tree(top[:1, :4], m, root[:1], L[:1], 1.0, 8, 2, 1, None)
+    assert t["n_nodes"][0] == 5
+    m[0, 2] = np.nextafter(np.float32(1.0), np.float32(0.0))
+    t = oracle.build_tree(top[:1, :4], m, root[:1], L[:1], 1.0, 8, 2, 1, None)
+    assert t["n_nodes"][0] == 6 and t["ufp_pos"][0, 0] == 2
+
+
+def test_tree_depth2_last_position_costs_one():
+    # Depth-2 repairs: the last position has no successor, so it costs one node
+    # and can still fit when the remaining budget is odd.
+    K = 4
+    top = np.array([[[10, 20], [11, 21], [12, 22], [13, 23]]])
+    margin = np.array([[0.1, 5, 5, 0.2]], dtype=np.float32)
+    redraft = np.array([[[50], [51], [52], [-1]]])
+    t = oracle.build_tree(top, margin, np.array([1]), np.array([30]), 1.0, 3, 2, 2, redraft)
+    assert t["n_nodes"][0] == 1 + K + 3
+    assert t["tok"][0, 5:8].tolist() == [20, 50, 23]
+    assert t["parent"][0, 5:8].tolist() == [0, 5, 3]
+    assert t["depth"][0, 5:8].tolist() == [1, 2, 4]
+
+
+# ---------------------------------------------------------------- S4 pins
+def _attn_case(seed, paged=False):
+    rng = np.random.default_rng(seed)
+    B, K, Hkv, G, D = 2, 4, 2, 3, 16
+    Hq = Hkv * G
+    top, margin, root, _, _, _, _, _, redraft = _random_case(seed, K=K, branches=3, budget=4, tau=1.0)
+    top, margin, root = top[:B], margin[:B], root[:B]
+    L = rng.integers(5, 40, size=B)
+    t = oracle.build_tree(top, margin, root, L, 1.0, 4, 3, 1)
+    N = 1 + K + 4
+    q = rng.standard_normal((B, N, Hq, D))
+    tk = rng.standard_normal((B, N, Hkv, D))
+    tv = rng.standard_normal((B, N, Hkv, D))
+    Lmax = int(L.max())
+    kc = rng.standard_normal((B, Lmax, Hkv, D))
+    vc = rng.standard_normal((B, Lmax, Hkv, D))
+    return q, tk, tv, kc, vc, L, t, D
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_tree_attn_equals_per_path_causal_sdpa(seed):
+    """Sec. 3.4: one tree pass equals separate causal attention per path."""
+    q, tk, tv, kc, vc, L, t, D = _attn_case(seed)
+    scale = 1.0 / math.sqrt(D)
+    out = oracle.tree_attn(q, tk, tv, kc, vc, L, t["n_nodes"], t["anc"], scale)
+    B, N, Hq, _ = q.shape
+    Hkv = tk.shape[2]
+    G = Hq // Hkv
+    for b in range(B):
+        for j in range(int(t["n_nodes"][b])):
+            # the path root..j as an explicit token sequence after the cache
+            path = []
+            x = j
+            while x >= 0:
+                path.append(x)
+                x = int(t["parent"][b, x])
+            path = path[::-1]
+            for h in range(Hq):
+                hk = h // G
+                ks = np.concatenate([kc[b, :L[b], hk], tk[b, path, hk]])
+                vs = np.concatenate([vc[b, :L[b], hk], tv[b, path, hk]])
+                # causal attention of the whole sequence; the last row is node j
+                Tq = torch.from_numpy(np.concatenate([np.zeros((len(ks) - 1, D)), q[b, j, h][None]]))
+                o = torch.nn.functional.scaled_dot_product_attention(
+                    Tq[None, None], torch.from_numpy(ks)[None, None], torch.from_numpy(vs)[None, None],
+                    is_causal=True, scale=scale)[0, 0, -1].numpy()
+                assert np.allclose(out[b, j, h], o, rtol=1e-11, atol=1e-12)
+
+
+def test_tree_attn_constant_keys_give_mean_of_values():
+    q, tk, tv, kc, vc, L, t, D = _attn_case(11)
+    kc[:] = 0.3
+    tk[:] = 0.3
+    out = oracle.tree_attn(q, tk, tv, kc, vc, L, t["n_nodes"], t["anc"], 0.25)
+    G = q.shape[2] // tk.shape[2]
+    for b in range(q.shape[0]):
+        for j in range(int(t["n_nodes"][b])):
+            vis = ancestors_by_parent_walk(t["parent"][b], j)
+            for h in range(q.shape[2]):
+                rows = [vc[b, i, h // G] for i in range(L[b])] + [tv[b, i, h // G] for i in sorted(vis)]
+                assert np.allclose(out[b, j, h], np.mean(rows, axis=0), rtol=1e-12, atol=1e-12)
+
+
+def test_tree_attn_paged_equals_contiguous():
+    q, tk, tv, kc, vc, L, t, D = _attn_case(5)
+    B, Lmax, Hkv, _ = kc.shape
+    ps = 4
+    npg = (Lmax + ps - 1) // ps
+    rng = np.random.default_rng(0)
+    perm = rng.permutation(B * npg)
+    table = perm.reshape(B, npg)
+    kp = np.zeros((B * npg, ps, Hkv, D))
+    vp = np.zeros((B * npg, ps, Hkv, D))
+    for b in range(B):
+        for s in range(Lmax):
+            kp[table[b, s // ps], s % ps] = kc[b, s]
+            vp[table[b, s // ps], s % ps] = vc[b, s]
+    a = oracle.tree_attn(q, tk, tv, kc, vc, L, t["n_nodes"], t["anc"], 0.25)
+    p = oracle.tree_attn(q, tk, tv, kp, vp, L, t["n_nodes"], t["anc"], 0.25, table, ps)
+    assert np.array_equal(a, p)
+
+
+# ---------------------------------------------------------------- S5 pins
+def _hand_accept(case):
+    g, t = _tree_hand()
+    c = g[case]
+    targ = np.array(c["targ"])[None]
+    r = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], g["K"])
+    return g, t, c, r
+
+
+@pytest.mark.parametrize("case", ["repair_win", "branch0_win"])
+def test_accept_hand(case):
+    g, t, c, r = _hand_accept(case)
+    for key in ("accept_len", "best_node", "diverge_depth"):
+        assert int(r[key][0]) == c[key], key
+    assert r["path_nodes"][0].tolist() == c["path_nodes"]
+    assert r["out_tokens"][0].tolist() == c["out_tokens"]
+
+
+def brute_force_accept(targ, n, tok, parent, depth):
+    """a(pi) for every root-to-leaf path, the maximum, and its first best leaf."""
+    children = {j: [] for j in range(n)}
+    for j in range(1, n):
+        children[int(parent[j])].append(j)
+    leaves = [j for j in range(n) if not children[j]]
+    best_a, best_nodes = -1, None
+    for leaf in leaves:
+        path = []
+        x = leaf
+        while x >= 0:
+            path.append(x)
+            x = int(parent[x])
+        path = path[::-1]
+        a = 0
+        for t in range(1, len(path)):
+            if tok[path[t]] == targ[path[t - 1]]:
+                a = t
+            else:
+                break
+        if a > best_a:
+            best_a = a
+    return best_a
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_accept_bruteforce_all_paths(seed):
+    top, margin, root, L, tau, budget, branches, d, redraft = _random_case(
+        seed, depth_rep=2 if seed % 2 else 1)
+    # a tiny token alphabet so that many nodes verify
+    top = top % 5
+    redraft = redraft % 5
+    for b in range(top.shape[0]):
+        for i in range(top.shape[1]):
+            top[b, i] = np.array([0, 1, 2, 3])   # distinct ranked ids per position
+    t = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft)
+    rng = np.random.default_rng(seed + 99)
+    targ = rng.integers(0, 3, size=t["tok"].shape)
+    r = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], top.shape[1])
+    for b in range(top.shape[0]):
+        n = int(t["n_nodes"][b])
+        a = brute_force_accept(targ[b], n, t["tok"][b], t["parent"][b], t["depth"][b])
+        assert r["accept_len"][b] == a
+        best = int(r["best_node"][b])
+        assert t["depth"][b, best] == a
+        # best is the lowest-index node at depth a whose path verifies
+        path = r["path_nodes"][b, :a + 1].tolist()
+        assert path[0] == 0 and path[-1] == best
+        for s in range(1, a + 1):
+            assert t["parent"][b, path[s]] == path[s - 1]
+            assert t["tok"][b, path[s]] == targ[b, path[s - 1]]
+        assert r["out_tokens"][b, :a + 1].tolist() == [int(t["tok"][b, x]) for x in path[1:]] + [int(targ[b, best])]
+        off = [s for s in range(a + 1) if path[s] > top.shape[1]]
+        assert r["diverge_depth"][b] == (off[0] if off else -1)
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_budget_zero_is_prefix_verification(seed):
+    """R = 0 leaves branch 0 alone: the result is plain prefix verification."""
+    w = W.WORKLOADS["tiny"].replace(vocab=64, budget=0, top_level=3.0)
+    d = W.draft_block(w, seed=seed)
+    x = W.bf16_to_f64(d.logits).reshape(-1, w.vocab)
+    ids, _, margin, _, _ = oracle.score_draft(x, w.topk)
+    K = w.block
+    t = oracle.build_tree(ids.reshape(1, K, -1), margin.astype(np.float32).reshape(1, K), d.root_tok,
+                          np.array([100]), w.tau, 0, w.branches, 1)
+    rng = np.random.default_rng(seed)
+    # the target agrees with the draft on a random prefix
+    e = int(rng.integers(0, K + 1))
+    targ = np.full((1, K + 1), -5)
+    targ[0, :e] = ids.reshape(K, -1)[:e, 0]
+    r = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], K)
+    # plain prefix verification written out: count leading draft tokens that
+    # equal the target's token at the previous position
+    draft = ids.reshape(K, -1)[:, 0]
+    a = 0
+    while a < K and draft[a] == targ[0, a]:
+        a += 1
+    assert r["accept_len"][0] == a == e
+    assert r["diverge_depth"][0] == -1
+    assert r["out_tokens"][0, :a + 1].tolist() == list(draft[:a]) + [int(targ[0, a])]
+
+
+# ---------------------------------------------------------------- S6 pins
+@pytest.mark.parametrize("case", ["repair_win", "branch0_win"])
+def test_resync_hand(case):
+    g, t, c, r = _hand_accept(case)
+    rng = np.random.default_rng(1)
+    N, Hkv, D, layers = 8, 2, 4, 3
+    tk = rng.standard_normal((layers, 1, N, Hkv, D))
+    tv = rng.standard_normal((layers, 1, N, Hkv, D))
+    kc = [rng.standard_normal((1, 120, Hkv, D)) for _ in range(layers)]
+    vc = [rng.standard_normal((1, 120, Hkv, D)) for _ in range(layers)]
+    k0 = [x.copy() for x in kc]
+    v0 = [x.copy() for x in vc]
+    s = oracle.resync(kc, vc, tk, tv, r["path_nodes"], r["accept_len"], r["diverge_depth"],
+                      r["out_tokens"], np.array([g["cache_len"]]), g["K"])
+    assert s["cache_len"][0] == c["cache_len"]
+    assert s["draft_valid_len"][0] == c["draft_valid_len"]
+    assert s["replay_tokens"][0].tolist() == c["replay_tokens"]
+    assert s["n_replay"][0] == c["n_replay"]
+    L, a = g["cache_len"], c["accept_len"]
+    for l in range(layers):
+        assert np.array_equal(kc[l][0, :L], k0[l][0, :L])            # older rows untouched
+        assert np.array_equal(kc[l][0, L + a + 1:], k0[l][0, L + a + 1:])
+        for tdep, node in enumerate(c["path_nodes"][:a + 1]):
+            assert np.array_equal(kc[l][0, L + tdep], tk[l, 0, node])
+            assert np.array_equal(vc[l][0, L + tdep], tv[l, 0, node])
+
+
+def test_resync_paged_matches_contiguous():
+    g, t, c, r = _hand_accept("repair_win")
+    rng = np.random.default_rng(2)
+    N, Hkv, D, ps = 8, 2, 4, 16
+    tk = rng.standard_normal((2, 1, N, Hkv, D))
+    tv = rng.standard_normal((2, 1, N, Hkv, D))
+    cont_k = [np.zeros((1, 128, Hkv, D)) for _ in range(2)]
+    cont_v = [np.zeros((1, 128, Hkv, D)) for _ in range(2)]
+    table = np.array([[5, 3, 7, 0, 6, 1, 2, 4]])
+    pag_k = [np.zeros((8, ps, Hkv, D)) for _ in range(2)]
+    pag_v = [np.zeros((8, ps, Hkv, D)) for _ in range(2)]
+    args = (tk, tv, r["path_nodes"], r["accept_len"], r["diverge_depth"], r["out_tokens"],
+            np.array([g["cache_len"]]), g["K"])
+    oracle.resync(cont_k, cont_v, *args)
+    oracle.resync(pag_k, pag_v, *args, block_table=table, page_size=ps)
+    for l in range(2):
+        for s in range(128):
+            assert np.array_equal(cont_k[l][0, s], pag_k[l][table[0, s // ps], s % ps])
+            assert np.array_equal(cont_v[l][0, s], pag_v[l][table[0, s // ps], s % ps])
+
+
+# ---------------------------------------------------------------- pin power
+def test_pins_catch_planted_mistakes():
+    """Plant typical mistakes in oracle outputs; the checkers must object."""
+    top, margin, root, L, tau, budget, branches, d, redraft = _random_case(4, K=8, budget=5, tau=2.0,
+                                                                            branches=3)
+    t = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft)
+    assert check_tree(t, top, margin, tau, budget, branches, d, L, redraft) == []
+    mutants = []
+    m = {k: v.copy() for k, v in t.items()}
+    m["parent"][0, 5] = m["parent"][0, 5] + 1         # wrong parent index
+    mutants.append(m)
+    m = {k: v.copy() for k, v in t.items()}
+    m["anc"][0, 3, 0] ^= np.uint64(1 << 1)             # dropped ancestor bit
+    mutants.append(m)
+    m = {k: v.copy() for k, v in t.items()}
+    m["tok"][0, 2] = top[0, 1, 1]                      # chain takes the rank-2 token
+    mutants.append(m)
+    m = {k: v.copy() for k, v in t.items()}
+    m["pos"][0, 4] += 1                                # off-by-one position
+    mutants.append(m)
+    for mt in mutants:
+        assert check_tree(mt, top, margin, tau, budget, branches, d, L, redraft) != []
+    # ascending order flipped (descending-margin admission) breaks the priority pin
+    flipped = oracle.build_tree(top, -margin + 3.0, root, L, tau, budget, branches, d, redraft)
+    assert check_tree(flipped, top, margin, tau, budget, branches, d, L, redraft) != []
+    # a non-strict gate (<=) admits margin == tau
+    m32 = np.full((1, 4), 1.0, dtype=np.float32)
+    t_le = oracle.build_tree(top[:1, :4], m32 - np.float32(1e-7), root[:1], L[:1], 1.0, 8, 2, 1)
+    assert check_tree(t_le, top[:1, :4], m32, 1.0, 8, 2, 1, L[:1]) != []
