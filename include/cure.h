@@ -1,0 +1,211 @@
+/*
+ * cure.h — C ABI of the CURE repair-verify step on one GB300 (sm_103a).
+ *
+ * CURE ("Local Uncertainty Repair for Block-Parallel Speculative Decoding")
+ * repairs a block-parallel draft at its low-margin positions and verifies the
+ * draft and the repairs in one tree pass.  One decoding step of the method is
+ * split into five calls, each one CUDA kernel (or two) on the caller's
+ * stream:
+ *
+ *   cure_score_draft  Sec. 3.3, Eq. (2)     top-k ids, margin, top-1 log-prob
+ *   cure_build_tree   Sec. 3.1 Eq. (1),     UFP gate + budgeted selection,
+ *                     Sec. 3.3, 3.4         flattened repair tree + ancestor mask
+ *   cure_tree_attn    Sec. 3.2, 3.4, 3.5    tree-masked GQA attention
+ *   cure_accept       Sec. 3.5 Eq. (4)      target argmax + longest accepted path
+ *   cure_resync_kv    Sec. 3.5, Alg. 1      write the path into the KV cache,
+ *                                           realign the draft state
+ *
+ * Conventions shared by every call
+ *  - Every pointer argument is a DEVICE pointer unless stated otherwise; the
+ *    caller owns all memory (inputs, outputs, caches, workspace).  The library
+ *    never allocates device memory.
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls are
+ *    asynchronous; nothing waits on the host.
+ *  - Arguments the host can check (sizes, null pointers, alignment) are
+ *    checked before anything is launched; a bad one returns
+ *    CURE_ERR_INVALID_ARG (or CURE_ERR_UNSUPPORTED for a valid but
+ *    unimplemented shape) and launches nothing.
+ *  - Conditions only the device can see (a cache slot past the capacity, a
+ *    missing or out-of-range page id, a node count past n_max) make the kernel
+ *    skip the offending access and raise a bit in a device error word;
+ *    cure_device_error() reads and clears it.
+ *  - Tensors are row-major, innermost dimension last.  bf16 is IEEE bfloat16.
+ *  - Tie rule everywhere: equal values rank the lower index first.
+ *  - Padding: entries of per-node outputs at j >= n_nodes[b] are -1 (ints) or
+ *    0 (ancestor words); output rows of cure_tree_attn at j >= n_nodes[b] are
+ *    left unwritten.
+ */
+#ifndef CURE_H_
+#define CURE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  CURE_OK = 0,
+  CURE_ERR_INVALID_ARG = 1,   /* a host-checkable argument is wrong; nothing launched */
+  CURE_ERR_CAPACITY = 2,      /* workspace too small for the shape; nothing launched */
+  CURE_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed */
+  CURE_ERR_DEVICE_FAULT = 4,  /* returned by cure_device_error when a kernel flagged bad data */
+  CURE_ERR_UNSUPPORTED = 5    /* valid but not implemented (e.g. head_dim != 128) */
+} cure_status;
+
+/* Bits of the device error word (cure_device_error). */
+#define CURE_DEVERR_PAGE      0x1   /* block_table entry < 0 or >= num_pages */
+#define CURE_DEVERR_SLOT      0x2   /* cache slot beyond the per-sequence capacity */
+#define CURE_DEVERR_NODES     0x4   /* n_nodes[b] outside [1, n_max] or a bad path/parent index */
+#define CURE_DEVERR_TOKEN     0x8   /* a token id outside [0, vocab) where one is required */
+
+/* Tree-construction parameters (Sec. 3.3 / 3.4 and Eq. 1). */
+typedef struct {
+  int32_t batch;         /* B, sequences */
+  int32_t block;         /* K, draft positions per block, 1..32 */
+  int32_t topk;          /* ranked candidates stored per position by cure_score_draft, 2..8 */
+  float tau;             /* margin threshold: position i is a UFP iff margin_i < tau (float32 compare) */
+  int32_t budget;        /* R, maximum repair nodes per sequence, >= 0; n_max = 1 + K + R <= 256 */
+  int32_t branches;      /* candidates per UFP counting the draft token: ranks 2..branches are
+                            the alternatives; 1..topk */
+  int32_t repair_depth;  /* 1: alternative leaf; 2: alternative + its re-drafted successor */
+  int32_t max_ufp;       /* 0 = no cap; else only the max_ufp lowest-margin UFPs are repaired */
+} cure_tree_params;
+
+/* KV-cache geometry (one layer). */
+typedef struct {
+  int32_t layout;        /* 0: contiguous [B][max_len][heads_kv][head_dim]
+                            1: paged [num_pages][page_size][heads_kv][head_dim] */
+  int32_t heads_kv;      /* Hkv */
+  int32_t head_dim;      /* D; 128 is implemented */
+  int32_t page_size;     /* paged: tokens per page (16); ignored when contiguous */
+  int32_t max_len;       /* contiguous: rows per sequence; paged: entries per block_table row */
+  int32_t num_pages;     /* paged: pages in the pool (bounds check); ignored when contiguous */
+  const int32_t* block_table; /* paged: device int32 [B][max_len] physical page ids; else NULL */
+} cure_kv_desc;
+
+/*
+ * Stage 1 — draft scores (Sec. 3.3, Eq. 2; Alg. 1 first step).
+ * For each of `rows` rows (B*K draft positions) of `vocab` bf16 logits:
+ *   top_ids[r][0..topk)  ids ranked by (logit desc, id asc)        int32
+ *   top_vals[r][0..topk) their logits widened to float32            float
+ *   margin[r]            top_vals[r][0] - top_vals[r][1] (Eq. 2; the log-softmax
+ *                        normaliser cancels, so it is also the log-prob gap)
+ *   logp1[r]             top_vals[r][0] - logsumexp(row)  (float32 accumulation)
+ * logits: bf16 [rows][vocab], any alignment.  2 <= topk <= 8, topk <= vocab.
+ * margin and logp1 may be NULL.  NaN logits are not supported (ranking undefined);
+ * -inf is allowed.
+ */
+cure_status cure_score_draft(const void* logits, int32_t rows, int32_t vocab, int32_t topk,
+                             int32_t* top_ids, float* top_vals, float* margin, float* logp1,
+                             void* stream);
+
+/*
+ * Stages 2+3 — UFP selection and repair-tree construction (Sec. 3.1 Eq. 1,
+ * Sec. 3.3, Sec. 3.4; Alg. 1 loop).  One warp per sequence.
+ * Inputs:  top_ids int32 [B][K][topk] and margin float [B][K] (from stage 1),
+ *          root_tok int32 [B] (last committed token), cache_len int32 [B] (L_b),
+ *          redraft int32 [B][K][branches-1]: the successor token of each
+ *          alternative when repair_depth == 2 (NULL otherwise).
+ * Selection: positions with margin < tau, in ascending (margin, position)
+ *   order; each alternative (i, r), r = 2..branches, costs min(repair_depth, K-i)
+ *   nodes and is admitted while the repair nodes stay <= budget (an alternative
+ *   that does not fit is skipped).
+ * Tree (n_max = 1 + K + budget nodes per sequence, W = ceil(n_max/64)):
+ *   node 0 root (root_tok, depth 0); nodes 1..K branch 0 (top-1 ids, chained);
+ *   then repair nodes in (i, r, depth) order: the rank-r id at position i as a
+ *   child of node i, and with depth-2 repairs (i < K-1) its successor.
+ * Outputs: n_nodes [B]; tok, pos (= L_b + depth), parent (-1 for the root),
+ *   depth: int32 [B][n_max]; anc uint64 [B][n_max][W] (bit a of node j set iff a
+ *   is on the root-to-j path, j included); ufp_pos int32 [B][K] (repaired
+ *   positions in selection order, then -1); n_ufp int32 [B].
+ * `p` is a HOST pointer.
+ */
+cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, const float* margin,
+                            const int32_t* root_tok, const int32_t* cache_len, const int32_t* redraft,
+                            int32_t* n_nodes, int32_t* tok, int32_t* pos, int32_t* parent,
+                            int32_t* depth, uint64_t* anc, int32_t* ufp_pos, int32_t* n_ufp,
+                            void* stream);
+
+/*
+ * Stage 4 — tree attention for one layer (Sec. 3.2 / 3.4 / 3.5: the target
+ * verifies every tree path in one pass).  For sequence b, node j < n_nodes[b],
+ * query head h (kv head h / (heads_q / heads_kv)):
+ *   out[b][j][h] = softmax(scale * q k^T) v over the cached keys 0..L_b-1 and
+ *                  the tree keys a with bit a of anc[b][j] set.
+ * q, out: bf16 [B][n_max][heads_q][D]; tree_k, tree_v: bf16 [B][n_max][heads_kv][D]
+ * (this step's target keys/values of the tree tokens); k_cache, v_cache: one
+ * layer in the layout of `kv` (a HOST pointer).  Accumulation is float32; the
+ * probabilities are rounded to bf16 before the PV product.  D = 128,
+ * heads_q % heads_kv == 0, all tensor base pointers 16-byte aligned.
+ * workspace: device scratch of at least cure_tree_attn_workspace_size() bytes,
+ * 256-byte aligned (split-KV partial results).
+ */
+cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v,
+                           const void* k_cache, const void* v_cache, const cure_kv_desc* kv,
+                           const int32_t* cache_len, const int32_t* n_nodes, const uint64_t* anc,
+                           int32_t batch, int32_t n_max, int32_t heads_q, float scale, void* out,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace cure_tree_attn needs for this shape (0 on a bad argument). */
+size_t cure_tree_attn_workspace_size(int32_t batch, int32_t n_max, int32_t heads_q,
+                                     const cure_kv_desc* kv);
+
+/*
+ * Stage 5 — acceptance walk (Sec. 3.5 Eq. 4, greedy decoding Sec. 4.1).
+ * targ[b][j] = argmax_v target_logits[b][j][v] (lowest id on ties) for
+ * j < n_nodes[b] (rows beyond are not read; their targ is -1).  Pass
+ * target_logits (bf16 [B][n_max][vocab]) to have the argmax computed, or
+ * target_logits = NULL and targ already filled with the target's tokens.
+ * A non-root node j is verified when tok[j] == targ[parent[j]]; it is accepted
+ * when every non-root node on its path is verified.  pi* = the deepest accepted
+ * node (lowest index on ties), a = its depth.
+ * Outputs (int32): accept_len [B] = a; best_node [B];
+ *   path_nodes [B][K+2]: path node at each depth 0..a, then -1;
+ *   out_tokens [B][K+2]: path tokens at depths 1..a, then targ[best] (the
+ *                        token after the path), then -1;
+ *   diverge_depth [B]: shallowest path depth whose node is a repair node
+ *                      (index > K), or -1 when branch 0 wins.
+ */
+cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch, int32_t n_max,
+                        int32_t vocab, int32_t block, const int32_t* n_nodes, const int32_t* tok,
+                        const int32_t* parent, const int32_t* depth, const uint64_t* anc,
+                        int32_t* accept_len, int32_t* best_node, int32_t* path_nodes,
+                        int32_t* out_tokens, int32_t* diverge_depth, void* stream);
+
+/*
+ * Stage 6 — repair resynchronisation (Sec. 3.5, Alg. 1 last step).
+ * For every layer l and sequence b, the K/V rows of the accepted path's nodes
+ * at depths 0..a are copied from tree_k/tree_v (bf16 [layers][B][n_max][Hkv][D])
+ * into cache slots L_b..L_b+a of k_caches[l]/v_caches[l] (layout `kv`).
+ * Then cache_len_out[b] = L_b + a + 1, draft_valid_len[b] = L_b + d when a
+ * repair path wins at divergence depth d (else L_b + a + 1), and
+ * replay_tokens[b] (int32 [B][K+2]) = the path tokens at depths d..a followed by
+ * the token after the path (only that token on branch-0 wins), then -1;
+ * n_replay[b] its length.  cache_len_out may alias cache_len_in.
+ * k_caches, v_caches: HOST arrays of `layers` device pointers (layers <= 128).
+ */
+cure_status cure_resync_kv(int32_t layers, void* const* k_caches, void* const* v_caches,
+                           const cure_kv_desc* kv, const void* tree_k, const void* tree_v,
+                           int32_t batch, int32_t n_max, int32_t block, const int32_t* path_nodes,
+                           const int32_t* accept_len, const int32_t* diverge_depth,
+                           const int32_t* out_tokens, const int32_t* cache_len_in,
+                           int32_t* cache_len_out, int32_t* draft_valid_len,
+                           int32_t* replay_tokens, int32_t* n_replay, void* stream);
+
+/* Reads and clears the device error word of the current device after
+ * synchronising `stream`.  *bits receives the CURE_DEVERR_* bits (may be NULL).
+ * Returns CURE_ERR_DEVICE_FAULT when any bit was set, CURE_OK otherwise. */
+cure_status cure_device_error(void* stream, int32_t* bits);
+
+/* Static description of a status code. */
+const char* cure_status_string(cure_status s);
+
+/* ABI version of this header (major * 100 + minor). */
+int32_t cure_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CURE_H_ */

@@ -1,0 +1,74 @@
+// Internal declarations shared by the translation units of libcure.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/cure.h"
+
+namespace cure {
+
+constexpr int kMaxNodes = 256;     // n_max limit: 4 ancestor words
+constexpr int kMaxLayers = 128;    // resync: layers passed by value
+
+// Device error word of the current device (see cure_device_error).
+int* device_error_word();
+int num_sms();
+
+__device__ __forceinline__ void flag(int* err, int bits) {
+  if (err) atomicOr(err, bits);
+}
+
+// ---- launchers (all asynchronous on `s`; return the launch's cudaError_t) ----
+cudaError_t launch_score(const uint16_t* logits, int64_t rows, int vocab, int topk,
+                         int32_t* top_ids, float* top_vals, float* margin, float* logp1,
+                         cudaStream_t s);
+// Target argmax over rows (b, j) with j < n_nodes[b]; other rows get -1.
+cudaError_t launch_target_argmax(const uint16_t* logits, int batch, int n_max, int vocab,
+                                 const int32_t* n_nodes, int32_t* targ, cudaStream_t s);
+
+cudaError_t launch_build_tree(const cure_tree_params& p, const int32_t* top_ids,
+                              const float* margin, const int32_t* root_tok,
+                              const int32_t* cache_len, const int32_t* redraft, int32_t* n_nodes,
+                              int32_t* tok, int32_t* pos, int32_t* parent, int32_t* depth,
+                              uint64_t* anc, int32_t* ufp_pos, int32_t* n_ufp, int* err,
+                              cudaStream_t s);
+
+cudaError_t launch_accept_walk(int batch, int n_max, int block, const int32_t* n_nodes,
+                               const int32_t* tok, const int32_t* parent, const int32_t* depth,
+                               const uint64_t* anc, const int32_t* targ, int32_t* accept_len,
+                               int32_t* best_node, int32_t* path_nodes, int32_t* out_tokens,
+                               int32_t* diverge_depth, int* err, cudaStream_t s);
+
+struct LayerPtrs {
+  void* k[kMaxLayers];
+  void* v[kMaxLayers];
+};
+
+cudaError_t launch_resync(int layers, const LayerPtrs& caches, const cure_kv_desc& kv,
+                          const uint16_t* tree_k, const uint16_t* tree_v, int batch, int n_max,
+                          int block, const int32_t* path_nodes, const int32_t* accept_len,
+                          const int32_t* diverge_depth, const int32_t* out_tokens,
+                          const int32_t* cache_len_in, int32_t* cache_len_out,
+                          int32_t* draft_valid_len, int32_t* replay_tokens, int32_t* n_replay,
+                          int* err, cudaStream_t s);
+
+// Tree attention: plan of the split-KV decomposition for a shape.
+struct AttnPlan {
+  int rows;        // query rows per (b, kv head) = n_max * G
+  int row_blocks;  // CTAs along the rows
+  int chunk;       // cache keys per split
+  int splits;      // splits per (b, kv head) at the maximum length
+  size_t ws_o;     // bytes of partial outputs
+  size_t ws_lse;   // bytes of partial log-sum-exps
+};
+bool plan_tree_attn(int batch, int n_max, int heads_q, const cure_kv_desc& kv, AttnPlan* plan);
+
+cudaError_t launch_tree_attn(const AttnPlan& plan, const uint16_t* q, const uint16_t* tree_k,
+                             const uint16_t* tree_v, const uint16_t* k_cache,
+                             const uint16_t* v_cache, const cure_kv_desc& kv,
+                             const int32_t* cache_len, const int32_t* n_nodes,
+                             const uint64_t* anc, int batch, int n_max, int heads_q, float scale,
+                             uint16_t* out, void* workspace, int* err, cudaStream_t s);
+
+}  // namespace cure

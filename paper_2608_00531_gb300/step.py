@@ -1,0 +1,97 @@
+"""One CURE repair-verify step over a batch, through the C ABI.
+
+``RepairVerifyStep`` owns the device buffers of every stage's outputs (and the
+tree-attention workspace) for a fixed shape, and runs the six stages in order
+on one stream:
+
+  score_draft -> build_tree -> tree_attn x layers -> accept -> resync_kv
+
+Inputs of a step (``StepInputs``) are the draft logits, the tree's target
+Q/K/V per layer and the target logits; the KV caches are persistent state
+owned by the caller.  Nothing here computes: every stage is a libcure call.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import List, Optional
+
+import torch
+
+from . import cure
+
+
+@dataclasses.dataclass
+class StepInputs:
+    draft_logits: torch.Tensor      # bf16 [B][K][V]
+    root_tok: torch.Tensor          # int32 [B]
+    cache_len: torch.Tensor         # int32 [B]
+    redraft: Optional[torch.Tensor]  # int32 [B][K][branches-1] or None
+    q: torch.Tensor                 # bf16 [layers][B][n_max][Hq][D]
+    tree_k: torch.Tensor            # bf16 [layers][B][n_max][Hkv][D]
+    tree_v: torch.Tensor            # bf16 [layers][B][n_max][Hkv][D]
+    target_logits: torch.Tensor     # bf16 [B][n_max][V]
+
+
+class RepairVerifyStep:
+    def __init__(self, batch: int, block: int, vocab: int, topk: int, tau: float, budget: int,
+                 branches: int, repair_depth: int, layers: int, heads_q: int, kv: cure.KVDesc,
+                 device: torch.device, max_ufp: int = 0, layer_map: Optional[List[int]] = None):
+        self.B, self.K, self.V, self.k = batch, block, vocab, topk
+        self.tau, self.R, self.branches, self.depth = tau, budget, branches, repair_depth
+        self.max_ufp = max_ufp
+        self.layers, self.Hq, self.kv = layers, heads_q, kv
+        self.n_max = 1 + block + budget
+        self.D = kv.head_dim
+        self.scale = 1.0 / float(self.D) ** 0.5
+        # logical layer -> physical cache index (aliasing when the caches of all
+        # layers do not fit in device memory)
+        self.layer_map = layer_map or list(range(layers))
+        dev = device
+        B, K, N = batch, block, self.n_max
+        W = (N + 63) // 64
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.score = (torch.empty(B, K, topk, **i32), torch.empty(B, K, topk, dtype=torch.float32, device=dev),
+                      torch.empty(B, K, dtype=torch.float32, device=dev),
+                      torch.empty(B, K, dtype=torch.float32, device=dev))
+        self.tree = dict(n_nodes=torch.empty(B, **i32), tok=torch.empty(B, N, **i32),
+                         pos=torch.empty(B, N, **i32), parent=torch.empty(B, N, **i32),
+                         depth=torch.empty(B, N, **i32),
+                         anc=torch.empty(B, N, W, dtype=torch.int64, device=dev),
+                         ufp_pos=torch.empty(B, K, **i32), n_ufp=torch.empty(B, **i32))
+        self.attn_out = torch.empty(layers, B, N, heads_q, self.D, dtype=torch.bfloat16, device=dev)
+        ws = cure.cure_tree_attn_workspace_size(B, N, heads_q, kv)
+        self.workspace = torch.empty(max(ws, 256), dtype=torch.uint8, device=dev)
+        self.targ = torch.empty(B, N, **i32)
+        P = K + 2
+        self.acc = dict(accept_len=torch.empty(B, **i32), best_node=torch.empty(B, **i32),
+                        path_nodes=torch.empty(B, P, **i32), out_tokens=torch.empty(B, P, **i32),
+                        diverge_depth=torch.empty(B, **i32))
+        self.rs = dict(draft_valid_len=torch.empty(B, **i32), replay_tokens=torch.empty(B, P, **i32),
+                       n_replay=torch.empty(B, **i32))
+        self.cache_len_out = torch.empty(B, **i32)
+
+    def run(self, x: StepInputs, k_caches: List[torch.Tensor], v_caches: List[torch.Tensor],
+            stream=None) -> dict:
+        ids, vals, margin, logp1 = cure.cure_score_draft(x.draft_logits, self.k, out=self.score,
+                                                         stream=stream)
+        tree = cure.cure_build_tree(ids, margin, x.root_tok, x.cache_len, self.tau, self.R,
+                                    self.branches, self.depth, x.redraft, self.max_ufp,
+                                    out=self.tree, stream=stream)
+        for l in range(self.layers):
+            p = self.layer_map[l]
+            cure.cure_tree_attn(x.q[l], x.tree_k[l], x.tree_v[l], k_caches[p], v_caches[p], self.kv,
+                                x.cache_len, tree["n_nodes"], tree["anc"], self.scale,
+                                out=self.attn_out[l], workspace=self.workspace, stream=stream)
+        acc = cure.cure_accept(tree, self.K, target_logits=x.target_logits, targ=self.targ,
+                               out=self.acc, stream=stream)
+        kl = [k_caches[self.layer_map[l]] for l in range(self.layers)]
+        vl = [v_caches[self.layer_map[l]] for l in range(self.layers)]
+        rs = cure.cure_resync_kv(kl, vl, self.kv, x.tree_k, x.tree_v, acc, x.cache_len, self.K,
+                                 cache_len_out=self.cache_len_out, out=self.rs, stream=stream)
+        return dict(score=self.score, tree=tree, attn=self.attn_out, acc=acc, resync=rs)
+
+    @property
+    def launches_per_step(self) -> int:
+        """Kernels one step launches: scan, tree, layers x (attention + reduce),
+        target argmax + walk, gather + finalize."""
+        return 1 + 1 + 2 * self.layers + 2 + 2

@@ -1,0 +1,120 @@
+"""Host-side checks of the C ABI that need no GPU.
+
+The library must load, export every function include/cure.h declares, and
+reject bad host arguments before launching anything.
+"""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cure.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__
+    try:
+        __graft_entry__.build()
+    except RuntimeError as e:  # no toolkit on this machine
+        pytest.skip(f"cannot build libcure: {e}")
+    from paper_2608_00531_gb300 import _lib
+    return _lib.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cure_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_five_stages():
+    names = declared_functions()
+    for n in ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_accept", "cure_resync_kv"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2608_00531_gb300 import _lib
+    out = subprocess.run(["nm", "-D", "--defined-only", _lib.LIB_PATH], capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\bT (cure_[a-z0-9_]+)$", out, flags=re.M))
+    for n in declared_functions():
+        assert n in exported, n
+        assert hasattr(lib, n)
+    assert set(_lib.EXPORTS) <= exported
+
+
+def test_version_and_status_strings(lib):
+    assert lib.cure_abi_version() == 100
+    assert lib.cure_status_string(0) == b"ok"
+    assert lib.cure_status_string(2) == b"workspace too small"
+
+
+def test_bad_arguments_are_rejected_on_the_host(lib):
+    from paper_2608_00531_gb300._lib import KVDesc, TreeParams
+    null = C.c_void_p(0)
+    # rows < 0, topk outside 2..8, topk > vocab
+    assert lib.cure_score_draft(null, -1, 100, 2, null, null, null, null, null) == 1
+    assert lib.cure_score_draft(null, 4, 100, 9, null, null, null, null, null) == 1
+    assert lib.cure_score_draft(null, 4, 2, 3, null, null, null, null, null) == 1
+    # zero rows is a no-op
+    assert lib.cure_score_draft(null, 0, 100, 2, null, null, null, null, null) == 0
+    # tree parameters
+    p = TreeParams(batch=2, block=33, topk=3, tau=1.0, budget=4, branches=2, repair_depth=1, max_ufp=0)
+    assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == 1
+    p.block, p.branches = 16, 4          # more branches than stored candidates
+    assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == 1
+    p.branches, p.budget = 3, 300       # n_max > 256
+    assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == 5
+    p.budget, p.batch = 4, 0            # empty batch: nothing to do
+    assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == 0
+    p.batch, p.repair_depth = 1, 2      # depth-2 repairs need the re-drafted successors
+    assert lib.cure_build_tree(C.byref(p), *([C.c_void_p(64)] * 5), null, *([C.c_void_p(64)] * 8), null) == 1
+    # attention: head_dim 64 unsupported, heads_q not a multiple of heads_kv
+    kv = KVDesc(layout=0, heads_kv=4, head_dim=64, page_size=16, max_len=100, num_pages=0, block_table=None)
+    assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 5
+    kv.head_dim = 128
+    assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 6, 1.0, null, null, 0, null) == 1
+    # paged without a block table
+    kv.layout = 1
+    assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 1
+    # resync: more layers than the ABI carries
+    kv.layout = 0
+    assert lib.cure_resync_kv(129, None, None, C.byref(kv), null, null, 1, 9, 8, *([null] * 9), null) == 1
+    # accept: n_max smaller than the chain
+    assert lib.cure_accept(null, null, 1, 4, 10, 8, *([null] * 10), null) == 1
+
+
+def test_workspace_size_is_a_host_computation(lib):
+    from paper_2608_00531_gb300._lib import KVDesc
+    kv = KVDesc(layout=0, heads_kv=4, head_dim=128, page_size=16, max_len=8192, num_pages=0, block_table=None)
+    n = lib.cure_tree_attn_workspace_size(32, 33, 28, C.byref(kv))
+    assert n > 0 and n % 4 == 0
+    # grows with the batch, zero on a bad shape
+    assert lib.cure_tree_attn_workspace_size(64, 33, 28, C.byref(kv)) == 2 * n
+    kv.head_dim = 96
+    assert lib.cure_tree_attn_workspace_size(32, 33, 28, C.byref(kv)) == 0
+
+
+def test_product_path_has_no_cpu_fallback():
+    """The binding fails loudly without the library and never imports the oracle."""
+    import importlib
+    import paper_2608_00531_gb300 as pkg
+    pkg_dir = os.path.dirname(pkg.__file__)
+    for fn in os.listdir(pkg_dir):
+        if fn.endswith(".py"):
+            src = open(os.path.join(pkg_dir, fn)).read()
+            assert "import oracle" not in src and "from oracle" not in src, fn
+    from paper_2608_00531_gb300 import _lib
+    saved, _lib._lib = _lib._lib, None
+    real = _lib.LIB_PATH
+    try:
+        _lib.LIB_PATH = real + ".missing"
+        with pytest.raises(ImportError):
+            _lib.load()
+    finally:
+        _lib.LIB_PATH = real
+        _lib._lib = saved

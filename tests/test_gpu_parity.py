@@ -1,0 +1,463 @@
+"""GPU parity: every stage through the C ABI against the CPU oracle.
+
+Bit-exact for ids, trees, accept results and resynced cache rows; margins
+bit-exact (the difference of two bf16 values is exact in float32); top-1
+log-probs within 1e-5 * max(1, |ref|); bf16 attention outputs within 2e-2
+absolute (and 2e-2 of the output scale on flat inputs).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_00531_gb300 import workload as W
+
+pytestmark = pytest.mark.gpu
+
+DEV = torch.device("cuda:0")
+ATTN_ABS_TOL = 2e-2
+LOGP_TOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def cure():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_00531_gb300 import cure as c
+    torch.cuda.set_device(DEV)
+    return c
+
+
+def _f64(t):
+    return W.bf16_to_f64(t)
+
+
+def _check_scores(c, logits_bf16, k, rows_sel=None):
+    ids, vals, margin, logp1 = c.cure_score_draft(logits_bf16.to(DEV), k)
+    torch.cuda.synchronize()
+    V = logits_bf16.shape[-1]
+    x = _f64(logits_bf16).reshape(-1, V)
+    sel = np.arange(x.shape[0]) if rows_sel is None else np.asarray(rows_sel)
+    o_ids, o_vals, o_m, _, o_lp = oracle.score_draft(x[sel], k)
+    g_ids = ids.cpu().numpy().reshape(-1, k)[sel]
+    g_vals = vals.cpu().numpy().reshape(-1, k)[sel]
+    g_m = margin.cpu().numpy().reshape(-1)[sel]
+    g_lp = logp1.cpu().numpy().reshape(-1)[sel]
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_vals, o_vals.astype(np.float32))
+    assert np.array_equal(g_m, o_m.astype(np.float32))
+    fin = np.isfinite(o_lp)
+    err = np.abs(g_lp[fin] - o_lp[fin])
+    assert np.all(err <= LOGP_TOL * np.maximum(1.0, np.abs(o_lp[fin]))), err.max()
+    return ids, margin, o_ids, o_m
+
+
+@pytest.mark.parametrize("name", ["tiny", "single8b"])
+def test_score_draft_workloads(cure, name):
+    w = W.WORKLOADS[name]
+    d = W.draft_block(w)
+    _check_scores(cure, d.logits, w.topk)
+
+
+@pytest.mark.parametrize("V,k,rows", [(1001, 2, 7), (32003, 3, 5), (77, 8, 33), (8, 2, 3), (9, 4, 4),
+                                      (151936, 4, 3), (40000, 5, 2)])
+def test_score_draft_ragged_and_ties(cure, V, k, rows):
+    rng = np.random.default_rng(V + k)
+    # a few distinct values: many exact ties, some -inf
+    x = rng.integers(-3, 4, size=(rows, V)).astype(np.float32) * 0.5
+    x[0, rng.integers(0, V, size=max(1, V // 10))] = -np.inf
+    _check_scores(cure, W.to_bf16(x), k)
+
+
+def test_score_draft_full_serve_shape_sampled(cure):
+    """batch 32 x block 16 x vocab 151936 in the launch configuration the
+    benchmark times; the oracle checks 64 sampled rows."""
+    w = W.WORKLOADS["serve32"]
+    d = W.draft_block(w)
+    rows = np.random.default_rng(0).choice(w.batch * w.block, size=64, replace=False)
+    _check_scores(cure, d.logits, w.topk, rows)
+
+
+def _tree_inputs(w, seed=None):
+    d = W.draft_block(w, seed=seed)
+    x = _f64(d.logits).reshape(-1, w.vocab)
+    o_ids, _, o_m, _, _ = oracle.score_draft(x, w.topk)
+    B, K, k = w.batch, w.block, w.topk
+    return d, o_ids.reshape(B, K, k), o_m.astype(np.float32).reshape(B, K)
+
+
+def _gpu_tree(c, ids, margin, root, L, w, redraft=None, max_ufp=0, tau=None, budget=None):
+    tau = w.tau if tau is None else tau
+    budget = w.budget if budget is None else budget
+    return c.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV),
+                             torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(root.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), tau, budget, w.branches,
+                             w.repair_depth,
+                             None if redraft is None else torch.from_numpy(redraft.astype(np.int32)).to(DEV),
+                             max_ufp)
+
+
+def _cmp_tree(g, t):
+    for key in ("n_nodes", "tok", "pos", "parent", "depth", "ufp_pos", "n_ufp"):
+        assert np.array_equal(g[key].cpu().numpy(), t[key]), key
+    assert np.array_equal(g["anc"].cpu().numpy().view(np.uint64), t["anc"])
+
+
+@pytest.mark.parametrize("name", ["tiny", "single8b", "serve32"])
+def test_build_tree_workloads(cure, name):
+    w = W.WORKLOADS[name]
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    g = _gpu_tree(cure, ids, margin, d.root_tok, L, w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, w.repair_depth)
+    _cmp_tree(g, t)
+
+
+def test_build_tree_depth2_long_shape(cure):
+    w = W.WORKLOADS["long64"].replace(vocab=4096)   # the tree does not depend on V
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    g = _gpu_tree(cure, ids, margin, d.root_tok, L, w, redraft=d.redraft)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, 2, d.redraft)
+    _cmp_tree(g, t)
+
+
+@pytest.mark.parametrize("budget", [0, 4, 8, 16, 32, 64])
+@pytest.mark.parametrize("tau", [0.25, 0.5, 1.0, 2.0, 4.0])
+def test_build_tree_sweep(cure, budget, tau):
+    w = W.WORKLOADS["sweep16"].replace(vocab=4096)
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    g = _gpu_tree(cure, ids, margin, d.root_tok, L, w, tau=tau, budget=budget)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, tau, budget, w.branches, 1)
+    _cmp_tree(g, t)
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_build_tree_random_params(cure, seed):
+    rng = np.random.default_rng(seed)
+    B, K = int(rng.integers(1, 9)), int(rng.integers(1, 33))
+    k = int(rng.integers(2, 9))
+    branches = int(rng.integers(1, k + 1))
+    depth = int(rng.integers(1, 3))
+    budget = int(rng.integers(0, 80))
+    tau = float(rng.choice([0.0, 0.5, 1.0, 3.0]))
+    max_ufp = int(rng.choice([0, 0, 1, 3]))
+    margin = (rng.integers(0, 16, size=(B, K)) * 0.25).astype(np.float32)
+    ids = rng.integers(0, 50000, size=(B, K, k))
+    root = rng.integers(0, 50000, size=B)
+    L = rng.integers(0, 1000, size=B)
+    redraft = rng.integers(0, 50000, size=(B, K, max(1, branches - 1)))
+    w = W.WORKLOADS["tiny"].replace(batch=B, block=K, branches=branches, repair_depth=depth)
+    g = cure.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV), torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(root.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), tau, budget, branches, depth,
+                             torch.from_numpy(redraft.astype(np.int32)).to(DEV), max_ufp)
+    t = oracle.build_tree(ids, margin, root, L, tau, budget, branches, depth, redraft, max_ufp)
+    _cmp_tree(g, t)
+
+
+# ------------------------------------------------------------------ attention
+def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0, branches=3):
+    rng = np.random.default_rng(seed)
+    k = max(2, branches)
+    margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
+    ids = rng.integers(0, 1000, size=(B, K, k))
+    root = rng.integers(0, 1000, size=B)
+    L = np.asarray(lens, dtype=np.int32)
+    t = oracle.build_tree(ids, margin, root, L, tau, budget, branches, 1)
+    N = 1 + K + budget
+    D = 128
+    q = W.normal_bf16((B, N, Hq, D), qk_std, rng)
+    tk = W.normal_bf16((B, N, Hkv, D), qk_std, rng)
+    tv = W.normal_bf16((B, N, Hkv, D), v_std, rng)
+    if paged:
+        table, npages = W.block_table(L, K, seed)
+        kc = W.normal_bf16((npages, 16, Hkv, D), qk_std, rng)
+        vc = W.normal_bf16((npages, 16, Hkv, D), v_std, rng)
+    else:
+        table, npages = None, 0
+        cap = int(L.max()) + K + 2
+        kc = W.normal_bf16((B, cap, Hkv, D), qk_std, rng)
+        vc = W.normal_bf16((B, cap, Hkv, D), v_std, rng)
+    return t, q, tk, tv, kc, vc, L, table, npages
+
+
+def _run_attn(c, t, q, tk, tv, kc, vc, L, table, npages, Hkv):
+    B = q.shape[0]
+    if table is not None:
+        bt = torch.from_numpy(table).to(DEV)
+        kv = c.kv_desc(Hkv, 128, table.shape[1], bt, 16, npages)
+    else:
+        kv = c.kv_desc(Hkv, 128, kc.shape[1])
+    out = c.cure_tree_attn(q.to(DEV), tk.to(DEV), tv.to(DEV), kc.to(DEV), vc.to(DEV), kv,
+                           torch.from_numpy(L).to(DEV),
+                           torch.from_numpy(t["n_nodes"].astype(np.int32)).to(DEV),
+                           torch.from_numpy(t["anc"].view(np.int64)).to(DEV), 1.0 / math.sqrt(128))
+    torch.cuda.synchronize()
+    assert c.cure_device_error() == 0
+    return out.float().cpu().numpy()
+
+
+def _cmp_attn(got, ref, t, seqs=None):
+    B = got.shape[0]
+    worst = 0.0
+    for b in (range(B) if seqs is None else seqs):
+        n = int(t["n_nodes"][b])
+        err = np.abs(got[b, :n] - ref[b, :n])
+        assert np.all(np.isfinite(got[b, :n]))
+        scale = max(1e-3, float(np.abs(ref[b, :n]).max()))
+        assert err.max() <= ATTN_ABS_TOL, err.max()
+        assert err.max() <= 2e-2 * scale, (err.max(), scale)
+        worst = max(worst, err.max())
+    return worst
+
+
+@pytest.mark.parametrize("paged", [False, True])
+@pytest.mark.parametrize("Hq,Hkv", [(8, 2), (28, 4), (32, 8)])
+@pytest.mark.parametrize("qk_std,v_std", [(1.0, 1.0), (2.0, 1.0), (1 / math.sqrt(128), 1 / math.sqrt(128))])
+def test_tree_attn_small(cure, paged, Hq, Hkv, qk_std, v_std):
+    # ragged lengths: empty cache, inside one tile, several tiles + tail, more than one split
+    lens = [0, 37, 700, 2100]
+    t, q, tk, tv, kc, vc, L, table, npages = _attn_case(4, 8, 6, Hq, Hkv, lens, paged, qk_std,
+                                                         v_std, seed=Hq + int(paged))
+    got = _run_attn(cure, t, q, tk, tv, kc, vc, L, table, npages, Hkv)
+    ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128), table, 16)
+    _cmp_attn(got, ref, t)
+
+
+def test_tree_attn_wide_tree_two_words(cure):
+    """n_max = 1 + 32 + 64 = 97 nodes: two ancestor words, two tree tiles."""
+    t, q, tk, tv, kc, vc, L, table, npages = _attn_case(2, 32, 64, 28, 4, [300, 1500], False, 1.0, 1.0,
+                                                         seed=7, tau=4.0)
+    assert t["n_nodes"].max() > 64
+    got = _run_attn(cure, t, q, tk, tv, kc, vc, L, table, npages, 4)
+    ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128))
+    _cmp_attn(got, ref, t)
+
+
+def test_tree_attn_full_serve_layer_sampled(cure):
+    """One layer at the benchmark's serving shape (batch 32, 28/4 heads, paged
+    16-token blocks, lengths U[1024, 8192]); the oracle checks 3 sequences."""
+    w = W.WORKLOADS["serve32"]
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, 1)
+    table, npages = W.block_table(L, w.block, w.seed)
+    rng = np.random.default_rng(3)
+    N, D = w.n_max, 128
+    q = W.normal_bf16((w.batch, N, w.heads_q, D), 1.0, rng)
+    tk = W.normal_bf16((w.batch, N, w.heads_kv, D), 1.0, rng)
+    tv = W.normal_bf16((w.batch, N, w.heads_kv, D), 1.0, rng)
+    g = torch.Generator(device=DEV).manual_seed(11)
+    kc = torch.randn(npages, 16, w.heads_kv, D, generator=g, device=DEV, dtype=torch.float32).to(torch.bfloat16)
+    vc = torch.randn(npages, 16, w.heads_kv, D, generator=g, device=DEV, dtype=torch.float32).to(torch.bfloat16)
+    bt = torch.from_numpy(table).to(DEV)
+    kv = cure.kv_desc(w.heads_kv, D, table.shape[1], bt, 16, npages)
+    out = cure.cure_tree_attn(q.to(DEV), tk.to(DEV), tv.to(DEV), kc, vc, kv, torch.from_numpy(L).to(DEV),
+                              torch.from_numpy(t["n_nodes"].astype(np.int32)).to(DEV),
+                              torch.from_numpy(t["anc"].view(np.int64)).to(DEV), 1.0 / math.sqrt(D))
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    got = out.float().cpu().numpy()
+    seqs = [int(np.argmax(t["n_nodes"])), int(np.argmax(L)), int(np.argmin(L))]
+    ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc.cpu()), _f64(vc.cpu()), L, t["n_nodes"],
+                           t["anc"], 1.0 / math.sqrt(D), table, 16, seqs=seqs)
+    _cmp_attn(got, ref, t, seqs)
+
+
+# ------------------------------------------------------------------ accept
+def _target_for(w, d, t, seed):
+    truth = W.target_truth(w, d, seed)
+    ids = W.synthetic_target_ids(truth, t["n_nodes"], t["tok"], t["parent"], t["depth"], w.vocab, seed)
+    return W.target_logits(ids, w.vocab, seed)
+
+
+def _gpu_tree_dict(t):
+    return {k: torch.from_numpy((v.view(np.int64) if k == "anc" else v.astype(np.int32))).to(DEV)
+            for k, v in t.items()}
+
+
+@pytest.mark.parametrize("name", ["tiny", "single8b", "serve32"])
+def test_accept_workloads(cure, name):
+    w = W.WORKLOADS[name]
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, 1)
+    tl = _target_for(w, d, t, w.seed)
+    acc = cure.cure_accept(_gpu_tree_dict(t), w.block, target_logits=tl.to(DEV))
+    targ_rows = _f64(tl).reshape(-1, w.vocab)
+    o_targ = oracle.row_argmax(targ_rows).reshape(w.batch, w.n_max)
+    o_acc = oracle.accept(o_targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], w.block)
+    g_targ = acc["targ"].cpu().numpy()
+    for b in range(w.batch):
+        n = int(t["n_nodes"][b])
+        assert np.array_equal(g_targ[b, :n], o_targ[b, :n])
+        assert (g_targ[b, n:] == -1).all()
+    for key in ("accept_len", "best_node", "path_nodes", "out_tokens", "diverge_depth"):
+        assert np.array_equal(acc[key].cpu().numpy(), o_acc[key]), key
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_accept_random_trees_with_ids(cure, seed):
+    """Random trees (depth-2 repairs included) with small-alphabet targets so
+    that many paths verify, through the precomputed-ids entry."""
+    rng = np.random.default_rng(seed)
+    B, K = 6, int(rng.integers(2, 20))
+    k, branches, depth = 4, 4, 1 + seed % 2
+    budget = int(rng.integers(0, 40))
+    margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
+    ids = np.tile(np.arange(k), (B, K, 1))
+    redraft = rng.integers(0, 3, size=(B, K, branches - 1))
+    t = oracle.build_tree(ids, margin, rng.integers(0, 3, size=B), rng.integers(0, 99, size=B), 1.5,
+                          budget, branches, depth, redraft)
+    targ = rng.integers(0, 3, size=t["tok"].shape)
+    o_acc = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], K)
+    acc = cure.cure_accept(_gpu_tree_dict(t), K, targ=torch.from_numpy(targ.astype(np.int32)).to(DEV))
+    for key in ("accept_len", "best_node", "path_nodes", "out_tokens", "diverge_depth"):
+        assert np.array_equal(acc[key].cpu().numpy(), o_acc[key]), key
+
+
+# ------------------------------------------------------------------ resync
+@pytest.mark.parametrize("paged", [False, True])
+def test_resync(cure, paged):
+    rng = np.random.default_rng(21 + int(paged))
+    B, K, budget, Hkv, D, layers = 5, 8, 6, 4, 128, 3
+    margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
+    ids = np.tile(np.arange(3), (B, K, 1))
+    t = oracle.build_tree(ids, margin, rng.integers(0, 3, size=B), rng.integers(0, 99, size=B), 1.5,
+                          budget, 3, 1)
+    targ = rng.integers(0, 3, size=t["tok"].shape)
+    o_acc = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], K)
+    L = rng.integers(0, 200, size=B).astype(np.int32)
+    N = 1 + K + budget
+    tk = W.normal_bf16((layers, B, N, Hkv, D), 1.0, rng)
+    tv = W.normal_bf16((layers, B, N, Hkv, D), 1.0, rng)
+    if paged:
+        table, npages = W.block_table(L, K, 5)
+        shape = (npages, 16, Hkv, D)
+        kv = cure.kv_desc(Hkv, D, table.shape[1], torch.from_numpy(table).to(DEV), 16, npages)
+    else:
+        table = None
+        shape = (B, int(L.max()) + K + 1, Hkv, D)
+        kv = cure.kv_desc(Hkv, D, shape[1])
+    kcs = [W.normal_bf16(shape, 1.0, rng) for _ in range(layers)]
+    vcs = [W.normal_bf16(shape, 1.0, rng) for _ in range(layers)]
+    kd = [x.to(DEV) for x in kcs]
+    vd = [x.to(DEV) for x in vcs]
+    acc = {k_: torch.from_numpy(v.astype(np.int32)).to(DEV) for k_, v in o_acc.items()}
+    rs = cure.cure_resync_kv(kd, vd, kv, tk.to(DEV), tv.to(DEV), acc, torch.from_numpy(L).to(DEV), K)
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    ko = [_f64(x) for x in kcs]
+    vo = [_f64(x) for x in vcs]
+    o_rs = oracle.resync(ko, vo, _f64(tk), _f64(tv), o_acc["path_nodes"], o_acc["accept_len"],
+                         o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, 16)
+    for key in ("cache_len", "draft_valid_len", "replay_tokens", "n_replay"):
+        assert np.array_equal(rs[key].cpu().numpy(), o_rs[key]), key
+    for l in range(layers):
+        assert np.array_equal(_f64(kd[l].cpu()), ko[l])
+        assert np.array_equal(_f64(vd[l].cpu()), vo[l])
+
+
+def test_resync_in_place_lengths(cure):
+    """cache_len_out may alias cache_len_in."""
+    B, K = 3, 4
+    acc = dict(accept_len=torch.tensor([0, 2, 4], dtype=torch.int32, device=DEV),
+               path_nodes=torch.tensor([[0, -1, -1, -1, -1, -1], [0, 1, 5, -1, -1, -1], [0, 1, 2, 3, 4, -1]],
+                                       dtype=torch.int32, device=DEV),
+               diverge_depth=torch.tensor([-1, 2, -1], dtype=torch.int32, device=DEV),
+               out_tokens=torch.tensor([[7, -1, -1, -1, -1, -1], [3, 9, 8, -1, -1, -1], [1, 2, 3, 4, 5, -1]],
+                                       dtype=torch.int32, device=DEV))
+    lens = torch.tensor([10, 20, 30], dtype=torch.int32, device=DEV)
+    kv = cure.kv_desc(4, 128, 64)
+    rs = cure.cure_resync_kv([], [], kv, None, None, acc, lens, K, cache_len_out=lens)
+    torch.cuda.synchronize()
+    assert lens.tolist() == [11, 23, 35]
+    assert rs["draft_valid_len"].tolist() == [11, 22, 35]
+    assert rs["n_replay"].tolist() == [1, 2, 1]
+    assert rs["replay_tokens"].cpu().numpy()[1, :2].tolist() == [9, 8]
+
+
+# ------------------------------------------------------------------ device-side checks
+def test_device_error_word_reports_bad_pages_and_slots(cure):
+    """Bad data the host cannot see: a missing page and a slot past the capacity.
+    The kernels skip the access and raise bits; the context stays usable."""
+    B, K, Hkv, D = 2, 4, 2, 128
+    acc = dict(accept_len=torch.tensor([1, 1], dtype=torch.int32, device=DEV),
+               path_nodes=torch.tensor([[0, 1, -1, -1, -1, -1]] * 2, dtype=torch.int32, device=DEV),
+               diverge_depth=torch.tensor([-1, -1], dtype=torch.int32, device=DEV),
+               out_tokens=torch.tensor([[1, 2, -1, -1, -1, -1]] * 2, dtype=torch.int32, device=DEV))
+    tk = torch.zeros(1, B, 1 + K, Hkv, D, dtype=torch.bfloat16, device=DEV)
+    table = torch.tensor([[0, -1], [1, 2]], dtype=torch.int32, device=DEV)
+    pages = torch.zeros(3, 16, Hkv, D, dtype=torch.bfloat16, device=DEV)
+    kv = cure.kv_desc(Hkv, D, 2, table, 16, 3)
+    assert cure.cure_device_error() == 0
+    # sequence 0 writes slots 16..17 (page entry -1); sequence 1 writes slots 40..41 (past 2 pages)
+    lens = torch.tensor([16, 40], dtype=torch.int32, device=DEV)
+    cure.cure_resync_kv([pages], [pages.clone()], kv, tk, tk.clone(), acc, lens, K)
+    bits = cure.cure_device_error()
+    assert bits & cure.DEVERR_PAGE and bits & cure.DEVERR_SLOT
+    assert cure.cure_device_error() == 0
+    # the context is still usable
+    x = torch.ones(4, device=DEV)
+    assert float(x.sum()) == 4.0
+
+
+# ------------------------------------------------------------------ whole step
+def test_full_step_serve_shape(cure):
+    """The six stages chained through RepairVerifyStep at the benchmark's shape
+    (2 layers); integers compared in full, attention on sampled sequences."""
+    from paper_2608_00531_gb300.step import RepairVerifyStep, StepInputs
+    w = W.WORKLOADS["serve32"]
+    layers = 2
+    d = W.draft_block(w)
+    L = W.cache_lengths(w)
+    x64 = _f64(d.logits).reshape(-1, w.vocab)
+    o_ids, _, o_m, _, _ = oracle.score_draft(x64, w.topk)
+    B, K, k, N = w.batch, w.block, w.topk, w.n_max
+    t = oracle.build_tree(o_ids.reshape(B, K, k), o_m.astype(np.float32).reshape(B, K), d.root_tok, L,
+                          w.tau, w.budget, w.branches, 1)
+    tl = _target_for(w, d, t, w.seed)
+    table, npages = W.block_table(L, K, w.seed)
+    rng = np.random.default_rng(9)
+    q = W.normal_bf16((layers, B, N, w.heads_q, 128), 1.0, rng)
+    tk = W.normal_bf16((layers, B, N, w.heads_kv, 128), 1.0, rng)
+    tv = W.normal_bf16((layers, B, N, w.heads_kv, 128), 1.0, rng)
+    g = torch.Generator(device=DEV).manual_seed(5)
+    kcs = [torch.randn(npages, 16, w.heads_kv, 128, generator=g, device=DEV).to(torch.bfloat16) for _ in range(layers)]
+    vcs = [torch.randn(npages, 16, w.heads_kv, 128, generator=g, device=DEV).to(torch.bfloat16) for _ in range(layers)]
+    seqs = [int(np.argmax(t["n_nodes"])), 5]
+    kc_host = [_f64(c.cpu()) for c in kcs]
+    vc_host = [_f64(c.cpu()) for c in vcs]
+    bt = torch.from_numpy(table).to(DEV)
+    kv = cure.kv_desc(w.heads_kv, 128, table.shape[1], bt, 16, npages)
+    st = RepairVerifyStep(B, K, w.vocab, k, w.tau, w.budget, w.branches, 1, layers, w.heads_q, kv, DEV)
+    xin = StepInputs(d.logits.to(DEV), torch.from_numpy(d.root_tok).to(DEV), torch.from_numpy(L).to(DEV),
+                     None, q.to(DEV), tk.to(DEV), tv.to(DEV), tl.to(DEV))
+    r = st.run(xin, kcs, vcs)
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    _cmp_tree(r["tree"], t)
+    for l in range(layers):
+        ref = oracle.tree_attn(_f64(q[l]), _f64(tk[l]), _f64(tv[l]), kc_host[l], vc_host[l], L, t["n_nodes"],
+                               t["anc"], 1.0 / math.sqrt(128), table, 16, seqs=seqs)
+        _cmp_attn(r["attn"][l].float().cpu().numpy(), ref, t, seqs)
+    o_targ = oracle.row_argmax(_f64(tl).reshape(-1, w.vocab)).reshape(B, N)
+    o_acc = oracle.accept(o_targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], K)
+    for key in ("accept_len", "best_node", "path_nodes", "out_tokens", "diverge_depth"):
+        assert np.array_equal(r["acc"][key].cpu().numpy(), o_acc[key]), key
+    o_rs = oracle.resync(kc_host, vc_host, _f64(tk), _f64(tv), o_acc["path_nodes"], o_acc["accept_len"],
+                         o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, 16)
+    for key in ("cache_len", "draft_valid_len", "replay_tokens", "n_replay"):
+        assert np.array_equal(r["resync"][key].cpu().numpy(), o_rs[key]), key
+    for l in range(layers):
+        assert np.array_equal(_f64(kcs[l].cpu()), kc_host[l])
+        assert np.array_equal(_f64(vcs[l].cpu()), vc_host[l])
