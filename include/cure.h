@@ -152,6 +152,36 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
 size_t cure_tree_attn_workspace_size(int32_t batch, int32_t n_max, int32_t heads_q,
                                      const cure_kv_desc* kv);
 
+/* Size of the static device scratch behind cure_tree_attn_noalloc (64 MiB). */
+#define CURE_NOALLOC_SCRATCH_BYTES (64u * 1024u * 1024u)
+
+/*
+ * cure_tree_attn without a caller-supplied workspace.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory — for instance a plugin in an inference server whose
+ * allocator owns (and has nearly filled) HBM, or a host framework that hands
+ * an extension only its input and output buffers.  It computes exactly what
+ * cure_tree_attn computes, with the same arguments minus the workspace; the
+ * split-KV partial results go to a 64 MiB array in the library's own static
+ * device memory, which every GPU that loads that part of the library keeps
+ * until the process exits.  It allocates nothing and calls no allocator.
+ *  - Shapes whose cure_tree_attn_workspace_size() is larger than
+ *    CURE_NOALLOC_SCRATCH_BYTES return CURE_ERR_CAPACITY and launch nothing.
+ *  - The first call on each device looks up the device address of the array
+ *    (cudaGetSymbolAddress); make that first call before any stream capture.
+ *  - All calls share the one array and it keeps the last call's contents.
+ *    Nothing in it needs to start at zero (each call writes every partial it
+ *    reads), but two calls that can overlap on the GPU — on unordered streams
+ *    or from different host threads — race on it and corrupt each other's
+ *    outputs: order such calls on one stream.
+ */
+cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k, const void* tree_v,
+                                   const void* k_cache, const void* v_cache,
+                                   const cure_kv_desc* kv, const int32_t* cache_len,
+                                   const int32_t* n_nodes, const uint64_t* anc, int32_t batch,
+                                   int32_t n_max, int32_t heads_q, float scale, void* out,
+                                   void* stream);
+
 /*
  * Stage 5 — acceptance walk (Sec. 3.5 Eq. 4, greedy decoding Sec. 4.1).
  * targ[b][j] = argmax_v target_logits[b][j][v] (lowest id on ties) for

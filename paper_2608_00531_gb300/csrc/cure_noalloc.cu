@@ -1,0 +1,90 @@
+// cure_tree_attn_noalloc: tree attention for callers that cannot allocate
+// device memory.
+//
+// Some callers only ever receive the buffers of their own inputs and outputs:
+// a plugin inside an inference server whose allocator has already reserved
+// nearly all of HBM for its KV cache, or a host framework that gives an
+// extension no allocator at all.  They cannot cudaMalloc the split-KV
+// workspace that cure_tree_attn takes.  This entry point runs the same kernels
+// with that workspace placed in a fixed array of the library's own static
+// device memory instead.
+//
+// The array below is CURE_NOALLOC_SCRATCH_BYTES (64 MiB).  Every GPU on which
+// this part of the library is loaded keeps it until the process exits.  In
+// host code `g_attn_scratch` is only a host-side stand-in for the symbol, not
+// a device address, so its device address is looked up once per device with
+// cudaGetSymbolAddress and that address is what the kernels receive.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_attn_scratch[CURE_NOALLOC_SCRATCH_BYTES];
+
+std::mutex g_scratch_mu;
+void* g_scratch_ptr[64];  // device address of g_attn_scratch, per device ordinal
+
+// Looks up (once per device, with that device current) the device address of
+// the scratch array.
+cudaError_t scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_attn_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+using namespace cure;
+
+extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k, const void* tree_v,
+                                              const void* k_cache, const void* v_cache,
+                                              const cure_kv_desc* kv, const int32_t* cache_len,
+                                              const int32_t* n_nodes, const uint64_t* anc,
+                                              int32_t batch, int32_t n_max, int32_t heads_q,
+                                              float scale, void* out, void* stream) {
+  if (!kv) return CURE_ERR_INVALID_ARG;
+  if (kv->layout != 0 && kv->layout != 1) return CURE_ERR_INVALID_ARG;
+  if (kv->heads_kv < 1 || kv->max_len < 0) return CURE_ERR_INVALID_ARG;
+  if (kv->head_dim != 128) return CURE_ERR_UNSUPPORTED;
+  if (kv->layout == 1 &&
+      (kv->page_size < 1 || kv->num_pages < 1 || !kv->block_table ||
+       (int64_t)kv->max_len * kv->page_size > INT32_MAX))
+    return CURE_ERR_INVALID_ARG;
+  if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
+    return CURE_ERR_INVALID_ARG;
+  if (n_max > kMaxNodes) return CURE_ERR_UNSUPPORTED;
+  if (batch == 0) return CURE_OK;
+  if (!q || !tree_k || !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out)
+    return CURE_ERR_INVALID_ARG;
+  const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(tree_k) |
+                        reinterpret_cast<uintptr_t>(tree_v) | reinterpret_cast<uintptr_t>(k_cache) |
+                        reinterpret_cast<uintptr_t>(v_cache) | reinterpret_cast<uintptr_t>(out);
+  if ((mis & 15) != 0 || (reinterpret_cast<uintptr_t>(anc) & 7) != 0) return CURE_ERR_INVALID_ARG;
+  AttnPlan plan;
+  if (!plan_tree_attn(batch, n_max, heads_q, *kv, &plan)) return CURE_ERR_INVALID_ARG;
+  if ((int64_t)batch * kv->heads_kv > 65535 || plan.splits > 65535) return CURE_ERR_UNSUPPORTED;
+  // the shape's split-KV partials must fit in the static array
+  if (plan.ws_o + plan.ws_lse > (size_t)CURE_NOALLOC_SCRATCH_BYTES) return CURE_ERR_CAPACITY;
+  void* scratch = nullptr;
+  if (scratch_address(&scratch) != cudaSuccess) return CURE_ERR_CUDA;
+  // Nothing in the scratch needs clearing: the reduce kernel reads only the
+  // partials that the attention kernel of this same call has written.
+  const cudaError_t e = launch_tree_attn(
+      plan, static_cast<const uint16_t*>(q), static_cast<const uint16_t*>(tree_k),
+      static_cast<const uint16_t*>(tree_v), static_cast<const uint16_t*>(k_cache),
+      static_cast<const uint16_t*>(v_cache), *kv, cache_len, n_nodes, anc, batch, n_max, heads_q,
+      scale, static_cast<uint16_t*>(out), scratch, device_error_word(),
+      static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? CURE_OK : CURE_ERR_CUDA;
+}
