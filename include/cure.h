@@ -59,6 +59,8 @@ typedef enum {
 #define CURE_DEVERR_SLOT      0x2   /* cache slot beyond the per-sequence capacity */
 #define CURE_DEVERR_NODES     0x4   /* n_nodes[b] outside [1, n_max] or a bad path/parent index */
 #define CURE_DEVERR_TOKEN     0x8   /* a token id outside [0, vocab) where one is required */
+#define CURE_DEVERR_TIMEOUT   0x10  /* a pipeline wait inside a kernel gave up (the CTA drained and left) */
+#define CURE_DEVERR_ALIGN     0x20  /* a kernel found its shared memory misaligned and did nothing */
 
 /* Tree-construction parameters (Sec. 3.3 / 3.4 and Eq. 1). */
 typedef struct {
@@ -79,7 +81,7 @@ typedef struct {
                             1: paged [num_pages][page_size][heads_kv][head_dim] */
   int32_t heads_kv;      /* Hkv */
   int32_t head_dim;      /* D; 128 is implemented */
-  int32_t page_size;     /* paged: tokens per page (16); ignored when contiguous */
+  int32_t page_size;     /* paged: tokens per page: 8, 16, 32 or 64; ignored when contiguous */
   int32_t max_len;       /* contiguous: rows per sequence; paged: entries per block_table row */
   int32_t num_pages;     /* paged: pages in the pool (bounds check); ignored when contiguous */
   const int32_t* block_table; /* paged: device int32 [B][max_len] physical page ids; else NULL */

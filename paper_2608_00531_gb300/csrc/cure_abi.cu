@@ -39,7 +39,14 @@ bool kv_ok(const cure_kv_desc* kv, cure_status* why) {
   }
   if (kv->layout == 1) {
     if (kv->page_size < 1 || kv->num_pages < 1 || !kv->block_table) return false;
-    if ((int64_t)kv->max_len * kv->page_size > INT32_MAX) return false;
+    if ((int64_t)kv->max_len * kv->page_size > INT32_MAX ||
+        (int64_t)kv->num_pages * kv->page_size > INT32_MAX)
+      return false;
+    // a page is whole TMA boxes of a 64-key tile
+    if (kv->page_size != 8 && kv->page_size != 16 && kv->page_size != 32 && kv->page_size != 64) {
+      *why = CURE_ERR_UNSUPPORTED;
+      return false;
+    }
   }
   return true;
 }

@@ -59,8 +59,12 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
   if (kv->head_dim != 128) return CURE_ERR_UNSUPPORTED;
   if (kv->layout == 1 &&
       (kv->page_size < 1 || kv->num_pages < 1 || !kv->block_table ||
-       (int64_t)kv->max_len * kv->page_size > INT32_MAX))
+       (int64_t)kv->max_len * kv->page_size > INT32_MAX ||
+       (int64_t)kv->num_pages * kv->page_size > INT32_MAX))
     return CURE_ERR_INVALID_ARG;
+  if (kv->layout == 1 && kv->page_size != 8 && kv->page_size != 16 && kv->page_size != 32 &&
+      kv->page_size != 64)
+    return CURE_ERR_UNSUPPORTED;
   if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
     return CURE_ERR_INVALID_ARG;
   if (n_max > kMaxNodes) return CURE_ERR_UNSUPPORTED;
