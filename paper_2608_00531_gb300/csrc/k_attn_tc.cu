@@ -44,8 +44,8 @@ constexpr int kOffK = kOffQ + 2 * kQHalf;
 constexpr int kOffV = kOffK + 2 * kTile;
 constexpr int kOffP = kOffV + 2 * kTile;
 constexpr int kOffBar = kOffP + BM * BN * 2;
-enum { B_KFULL = 0, B_VFULL = 2, B_KVEMPTY = 4, B_SFULL = 6, B_SFREE = 8, B_PFULL = 10,
-       B_PVDONE = 11, B_DRAIN = 12, kNumBars = 13 };
+enum { B_KFULL = 0, B_VFULL = 2, B_KEMPTY = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
+       B_PFULL = 12, B_PVDONE = 13, B_DRAIN = 14, kNumBars = 15 };
 constexpr int kOffTmemSlot = kOffBar + 8 * kNumBars;
 constexpr int kOffAbort = kOffTmemSlot + 4;
 constexpr int kSmemBytes = kOffBar + 128;
@@ -135,7 +135,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar(B_KFULL + i), 1);
       mbar_init(bar(B_VFULL + i), 1);
-      mbar_init(bar(B_KVEMPTY + i), 1);
+      mbar_init(bar(B_KEMPTY + i), 1);
+      mbar_init(bar(B_VEMPTY + i), 1);
       mbar_init(bar(B_SFULL + i), 1);
       mbar_init(bar(B_SFREE + i), 128);
     }
@@ -174,60 +175,86 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
 
   if (warp == 4) {
     // ------------------------------------------------------------ TMA producer
-    int issued = 0;
-    for (int j = 0; j < n_tiles; ++j) {
-      const int s = j & 1;
-      const uint32_t use = (uint32_t)j >> 1;
-      if (!wait_warp(bar(B_KVEMPTY + s), (use & 1u) ^ 1u, abort_flag, A.err)) break;
-      if (lane == 0) {
-        const uint32_t dk = sb + kOffK + s * kTile, dv = sb + kOffV + s * kTile;
-        mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
-        mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
-        if (j < n_cache_tiles) {
-          const int t0 = key_beg + j * BN;
-          if (A.kv.layout == 0) {
-            const int row = b * A.kv.max_len + t0;
-            for (int hf = 0; hf < 2; ++hf) {
-              tma_load_3d(dk + hf * kKVHalf, &tm_k, bar(B_KFULL + s), hf * 64, h, row);
-              tma_load_3d(dv + hf * kKVHalf, &tm_v, bar(B_VFULL + s), hf * 64, h, row);
-            }
-          } else {
-            const int ps = A.kv.page_size;
-            for (int p = 0; p < BN / ps; ++p) {
-              const int tok = t0 + p * ps;
-              int page = -1;
-              if (tok < key_end) {
-                page = A.kv.block_table[(int64_t)b * A.kv.max_len + tok / ps];
-                if (page < 0 || page >= A.kv.num_pages) {
-                  flag(A.err, CURE_DEVERR_PAGE);
-                  page = -1;  // a box wholly out of bounds reads zeros
-                }
-              }
-              for (int hf = 0; hf < 2; ++hf) {
-                tma_load_3d(dk + hf * kKVHalf + p * ps * 128, &tm_k, bar(B_KFULL + s), hf * 64, h,
-                            page * ps);
-                tma_load_3d(dv + hf * kKVHalf + p * ps * 128, &tm_v, bar(B_VFULL + s), hf * 64, h,
-                            page * ps);
-              }
-            }
-          }
-        } else {
-          const int row = b * A.n_max + (j - n_cache_tiles) * BN;
-          for (int hf = 0; hf < 2; ++hf) {
-            tma_load_3d(dk + hf * kKVHalf, &tm_tk, bar(B_KFULL + s), hf * 64, h, row);
-            tma_load_3d(dv + hf * kKVHalf, &tm_tv, bar(B_VFULL + s), hf * 64, h, row);
+    // One 64-key tile of K (or V) into `dst`: cache tiles come from the
+    // contiguous or paged cache, the tree tiles from this step's tree rows.
+    // Physical page ids of the split are fetched 32 tiles at a time, one tile
+    // per lane (up to 8 pages of a 64-key tile in registers), and handed to
+    // lane 0 by shuffles: no dependent global load sits in front of a copy.
+    const int ps = A.kv.page_size;
+    const int ppt = A.kv.layout == 1 ? BN / ps : 0;  // pages per tile
+    int pg[8];
+    auto fetch_pages = [&](int window) {
+      const int j = window * 32 + lane;
+#pragma unroll
+      for (int p = 0; p < 8; ++p) {
+        pg[p] = -1;
+        if (p < ppt && j < n_cache_tiles) {
+          const int tok = key_beg + j * BN + p * ps;
+          if (tok < key_end) {
+            const int page = A.kv.block_table[(int64_t)b * A.kv.max_len + tok / ps];
+            if (page < 0 || page >= A.kv.num_pages) flag(A.err, CURE_DEVERR_PAGE);
+            else pg[p] = page;  // a missing page stays -1: its box reads zeros
           }
         }
       }
+    };
+    int tile_pg[8];
+    // One 64-key tile of K (or V) into `dst`: cache tiles come from the
+    // contiguous or paged cache, the tree tiles from this step's tree rows.
+    auto load_tile = [&](int j, uint32_t dst, uint32_t fb, const CUtensorMap* cache_map,
+                         const CUtensorMap* tree_map) {
+      if (j < n_cache_tiles) {
+        const int t0 = key_beg + j * BN;
+        if (A.kv.layout == 0) {
+          const int row = b * A.kv.max_len + t0;
+          for (int hf = 0; hf < 2; ++hf) tma_load_3d(dst + hf * kKVHalf, cache_map, fb, hf * 64, h, row);
+        } else {
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {
+            if (p < ppt) {
+              for (int hf = 0; hf < 2; ++hf)
+                tma_load_3d(dst + hf * kKVHalf + p * ps * 128, cache_map, fb, hf * 64, h,
+                            tile_pg[p] * ps);
+            }
+          }
+        }
+      } else {
+        const int row = b * A.n_max + (j - n_cache_tiles) * BN;
+        for (int hf = 0; hf < 2; ++hf) tma_load_3d(dst + hf * kKVHalf, tree_map, fb, hf * 64, h, row);
+      }
+    };
+    int k_issued = 0, v_issued = 0;
+    for (int j = 0; j < n_tiles; ++j) {
+      const int s = j & 1;
+      const uint32_t use = (uint32_t)j >> 1;
+      if (ppt > 0 && j < n_cache_tiles) {
+        if ((j & 31) == 0) fetch_pages(j >> 5);
+#pragma unroll
+        for (int p = 0; p < 8; ++p) tile_pg[p] = __shfl_sync(0xffffffffu, pg[p], j & 31);
+      }
+      // K stage s frees when S(j-2) completes, V stage s when PV(j-2) does
+      if (!wait_warp(bar(B_KEMPTY + s), (use & 1u) ^ 1u, abort_flag, A.err)) break;
+      if (lane == 0) {
+        const uint32_t dk = sb + kOffK + s * kTile;
+        mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
+        load_tile(j, dk, bar(B_KFULL + s), &tm_k, &tm_tk);
+      }
       __syncwarp();
-      issued = j + 1;
+      k_issued = j + 1;
+      if (!wait_warp(bar(B_VEMPTY + s), (use & 1u) ^ 1u, abort_flag, A.err)) break;
+      if (lane == 0) {
+        const uint32_t dv = sb + kOffV + s * kTile;
+        mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
+        load_tile(j, dv, bar(B_VFULL + s), &tm_v, &tm_tv);
+      }
+      __syncwarp();
+      v_issued = j + 1;
     }
     if (*abort_flag) {  // let copies in flight land before the CTA's smem goes away
-      for (int jj = max(0, issued - 2); jj < issued; ++jj) {
-        const uint32_t par = ((uint32_t)jj >> 1) & 1u;
-        wait_bounded(bar(B_KFULL + (jj & 1)), par, abort_flag, A.err, false);
-        wait_bounded(bar(B_VFULL + (jj & 1)), par, abort_flag, A.err, false);
-      }
+      for (int jj = max(0, k_issued - 2); jj < k_issued; ++jj)
+        wait_bounded(bar(B_KFULL + (jj & 1)), ((uint32_t)jj >> 1) & 1u, abort_flag, A.err, false);
+      for (int jj = max(0, v_issued - 2); jj < v_issued; ++jj)
+        wait_bounded(bar(B_VFULL + (jj & 1)), ((uint32_t)jj >> 1) & 1u, abort_flag, A.err, false);
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------ MMA issuer
@@ -249,13 +276,13 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
                       sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
         }
         mma_commit(bar(B_SFULL + s));
+        mma_commit(bar(B_KEMPTY + s));
       }
       __syncwarp();
       return true;
     };
-    bool ok = issue_s(0);
+    bool ok = issue_s(0) && (n_tiles < 2 || issue_s(1));
     for (int j = 0; ok && j < n_tiles; ++j) {
-      if (j + 1 < n_tiles && !issue_s(j + 1)) break;
       const int s = j & 1;
       const uint32_t use = (uint32_t)j >> 1;
       if (!wait_warp(bar(B_PFULL), (uint32_t)j & 1u, abort_flag, A.err)) break;
@@ -270,9 +297,11 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
                       (j > 0 || ks > 0) ? 1u : 0u);
         }
         mma_commit(bar(B_PVDONE));
-        mma_commit(bar(B_KVEMPTY + s));
+        mma_commit(bar(B_VEMPTY + s));
       }
       __syncwarp();
+      // S(j+2) reuses the S buffer that softmax(j) has finished reading
+      if (j + 2 < n_tiles && !issue_s(j + 2)) break;
     }
     // every MMA issued by this warp has completed once the drain barrier flips
     if (lane == 0) mma_commit(bar(B_DRAIN));
@@ -327,11 +356,26 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           x[32 + i] = 32 + i < lim ? __uint_as_float(u1[i]) * c : -INFINITY;
         }
       }
-      float mt = -INFINITY;
+      float mx[8];
 #pragma unroll
-      for (int i = 0; i < 64; ++i) mt = fmaxf(mt, x[i]);
+      for (int i = 0; i < 8; ++i) mx[i] = x[i];
+#pragma unroll
+      for (int i = 8; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], x[i]);
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       const float m_new = fmaxf(m_run, mt);
       const bool need = m_new > m_run + 8.0f;
+      // the row max used for this tile's probabilities (lazily updated)
+      const float m_use = need ? m_new : m_run;
+      const float base = m_use == -INFINITY ? 0.f : m_use;
+      uint32_t pk[32];
+      float sm[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float p0 = ex2(x[2 * i] - base), p1 = ex2(x[2 * i + 1] - base);
+        sm[i & 3] += p0 + p1;
+        pk[i] = pack_bf16(p0, p1);
+      }
 
       // P and O are free once the previous PV product has completed
       if (j > 0) {
@@ -358,16 +402,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         l_run *= ex2(m_run - m_new);
         m_run = m_new;
       }
-      const float base = m_run == -INFINITY ? 0.f : m_run;
-      uint32_t pk[32];
-      float sum = 0.f;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float p0 = ex2(x[2 * i] - base), p1 = ex2(x[2 * i + 1] - base);
-        sum += p0 + p1;
-        pk[i] = pack_bf16(p0, p1);
-      }
-      l_run += sum;
+      l_run += (sm[0] + sm[1]) + (sm[2] + sm[3]);
       const uint32_t prow = sb + kOffP + row * 128;
 #pragma unroll
       for (int q = 0; q < 8; ++q)
