@@ -353,7 +353,7 @@ def main():
     else:
         roof = {"bound": "tensor", "achieved": round(attn_tflops, 1), "peak": pk["bf16_tflops_sustained"],
                 "unit": "TFLOP/s", "frac": round(attn_tflops / pk["bf16_tflops_sustained"], 4)}
-    roof.update({"traffic": None, "kernel": "tree attention (tree_attn_tc_kernel + split-KV reduce), per layer",
+    roof.update({"traffic": None, "kernel": "tree attention (tree_attn_tc_kernel, persistent, split units merged in-kernel), per layer",
                  "algorithmic_bytes_per_launch": alg["attn_bytes"],
                  "algorithmic_flops_per_launch": alg["attn_flops"], "avg_launch_ms": round(attn_avg, 4),
                  "peak_source": pk["source"] + " (MEASURED_PEAKS.json hbm_gbs)"})

@@ -15,10 +15,12 @@ struct AttnArgs {
   const int32_t* cache_len;
   const int32_t* n_nodes;
   const uint64_t* anc;
-  int batch, n_max, heads_q, G, W, chunk, splits, rows_pad, cap;
+  int batch, n_max, heads_q, G, W, cap;
+  int units_max;   // piece counters in the workspace
   float scale_log2;
-  float* ws_o;
-  float* ws_lse;
+  int* cnt;        // [units_max] pieces of each unit merged so far (zero between launches)
+  float* ws_o;     // [(units_max + kAttnMaxCtas) * 256][128] partial outputs
+  float* ws_lse;   // [(units_max + kAttnMaxCtas) * 256] partial base-2 log-sum-exps
   uint16_t* out;
   int* err;
 };
@@ -26,8 +28,10 @@ struct AttnArgs {
 constexpr int kAttnD = 128;       // head dim
 constexpr int kAttnRowsCta = 128; // query rows (node x group head) per CTA
 constexpr int kAttnKeys = 64;     // keys per tile
+constexpr int kAttnMaxBatch = 256;  // sequences per call (the CTA keeps per-sequence prefix sums)
+constexpr int kAttnMaxCtas = 256;   // persistent CTAs (one per SM, at most this many)
 
-// Main split-KV kernel on tcgen05 tensor cores: partial (O, lse) per row.
+// The persistent tcgen05 kernel (writes `out`; merges split units itself).
 cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s);
 
 }  // namespace cure

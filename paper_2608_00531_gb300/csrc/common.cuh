@@ -10,6 +10,7 @@ namespace cure {
 
 constexpr int kMaxNodes = 256;     // n_max limit: 4 ancestor words
 constexpr int kMaxLayers = 128;    // resync: layers passed by value
+constexpr int kAttnBatchLimit = 256;  // tree attention: sequences per call
 
 // Device error word of the current device (see cure_device_error).
 int* device_error_word();
@@ -53,14 +54,13 @@ cudaError_t launch_resync(int layers, const LayerPtrs& caches, const cure_kv_des
                           int32_t* draft_valid_len, int32_t* replay_tokens, int32_t* n_replay,
                           int* err, cudaStream_t s);
 
-// Tree attention: plan of the split-KV decomposition for a shape.
+// Tree attention: workspace layout for a shape.
 struct AttnPlan {
-  int rows;        // query rows per (b, kv head) = n_max * G
-  int row_blocks;  // CTAs along the rows
-  int chunk;       // cache keys per split
-  int splits;      // splits per (b, kv head) at the maximum length
+  int units_max;   // (sequence, kv head, row group) units at n_max
+  size_t ws_cnt;   // bytes of per-unit piece counters (256-byte rounded)
   size_t ws_o;     // bytes of partial outputs
   size_t ws_lse;   // bytes of partial log-sum-exps
+  size_t total() const { return ws_cnt + ws_o + ws_lse; }
 };
 bool plan_tree_attn(int batch, int n_max, int heads_q, const cure_kv_desc& kv, AttnPlan* plan);
 

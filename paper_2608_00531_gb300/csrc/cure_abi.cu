@@ -134,7 +134,7 @@ size_t cure_tree_attn_workspace_size(int32_t batch, int32_t n_max, int32_t heads
   if (batch < 0 || n_max < 1 || n_max > kMaxNodes || heads_q < 1 || !kv_ok(kv, &why)) return 0;
   AttnPlan plan;
   if (!plan_tree_attn(batch, n_max, heads_q, *kv, &plan)) return 0;
-  return plan.ws_o + plan.ws_lse;
+  return plan.total();
 }
 
 cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v,
@@ -146,7 +146,8 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
   if (!kv_ok(kv, &why)) return why;
   if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
     return CURE_ERR_INVALID_ARG;
-  if (n_max > kMaxNodes) return CURE_ERR_UNSUPPORTED;
+  if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
+    return CURE_ERR_UNSUPPORTED;
   if (batch == 0) return CURE_OK;
   if (!q || !tree_k || !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out ||
       !workspace)
@@ -156,8 +157,7 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
     return CURE_ERR_INVALID_ARG;
   AttnPlan plan;
   if (!plan_tree_attn(batch, n_max, heads_q, *kv, &plan)) return CURE_ERR_INVALID_ARG;
-  if ((int64_t)batch * kv->heads_kv > 65535 || plan.splits > 65535) return CURE_ERR_UNSUPPORTED;
-  if (workspace_bytes < plan.ws_o + plan.ws_lse) return CURE_ERR_CAPACITY;
+  if (workspace_bytes < plan.total()) return CURE_ERR_CAPACITY;
   return from_cuda(launch_tree_attn(plan, static_cast<const uint16_t*>(q),
                                     static_cast<const uint16_t*>(tree_k),
                                     static_cast<const uint16_t*>(tree_v),

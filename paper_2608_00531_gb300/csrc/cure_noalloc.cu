@@ -67,7 +67,8 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
     return CURE_ERR_UNSUPPORTED;
   if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
     return CURE_ERR_INVALID_ARG;
-  if (n_max > kMaxNodes) return CURE_ERR_UNSUPPORTED;
+  if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
+    return CURE_ERR_UNSUPPORTED;
   if (batch == 0) return CURE_OK;
   if (!q || !tree_k || !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out)
     return CURE_ERR_INVALID_ARG;
@@ -77,13 +78,13 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
   if ((mis & 15) != 0 || (reinterpret_cast<uintptr_t>(anc) & 7) != 0) return CURE_ERR_INVALID_ARG;
   AttnPlan plan;
   if (!plan_tree_attn(batch, n_max, heads_q, *kv, &plan)) return CURE_ERR_INVALID_ARG;
-  if ((int64_t)batch * kv->heads_kv > 65535 || plan.splits > 65535) return CURE_ERR_UNSUPPORTED;
   // the shape's split-KV partials must fit in the static array
-  if (plan.ws_o + plan.ws_lse > (size_t)CURE_NOALLOC_SCRATCH_BYTES) return CURE_ERR_CAPACITY;
+  if (plan.total() > (size_t)CURE_NOALLOC_SCRATCH_BYTES) return CURE_ERR_CAPACITY;
   void* scratch = nullptr;
   if (scratch_address(&scratch) != cudaSuccess) return CURE_ERR_CUDA;
-  // Nothing in the scratch needs clearing: the reduce kernel reads only the
-  // partials that the attention kernel of this same call has written.
+  // The call zeroes the piece counters at the front of the scratch itself (an
+  // asynchronous memset on the stream); every partial that is read back was
+  // written earlier in the same call.
   const cudaError_t e = launch_tree_attn(
       plan, static_cast<const uint16_t*>(q), static_cast<const uint16_t*>(tree_k),
       static_cast<const uint16_t*>(tree_v), static_cast<const uint16_t*>(k_cache),

@@ -1,20 +1,28 @@
-// Stage 4 main kernel: tree-masked GQA attention on tcgen05 tensor cores
-// (Sec. 3.2 / 3.4 / 3.5, Tree Attention).
+// Stage 4: tree-masked GQA attention on tcgen05 tensor cores (Sec. 3.2 / 3.4 /
+// 3.5, Tree Attention), one persistent CTA per SM.
 //
-// One CTA = 128 query rows (packed (node, group head) pairs of one sequence and
-// kv head) x one split of the cache keys (plus the tree keys on the last
-// split).  Six warps:
-//   warps 0-3  softmax: thread t owns query row t = TMEM lane t
-//   warp 4     TMA producer: 64-key K and V tiles, 128-byte swizzled,
-//              double-buffered
-//   warp 5     MMA issuer (one lane): S = Q K^T (M128 N64 K128) into one of two
-//              TMEM S buffers, O += P V (M128 N128 K64) into the TMEM O buffer
-// TMEM: S[2] (2 x 64 columns) + O (128 columns) = 256 columns, so two CTAs
-// share an SM.  P goes through swizzled shared memory.  The online softmax
-// keeps a lazily updated row max: O in TMEM is rescaled only when the max
-// grows by more than 2^8, which keeps every probability below 256.
-// Every wait on an mbarrier is bounded; on a timeout the CTA raises
-// CURE_DEVERR_TIMEOUT, drains its copies and MMAs, frees TMEM and leaves.
+// Work.  A unit is (sequence b, kv head h, row group rg): up to 256 query rows,
+// the packed (node, group head) pairs of 2 * npb tree nodes (npb = 128 / G
+// nodes per 128-row M tile).  A unit's keys are cut into 64-key tiles: the
+// cache tiles 0..ceil(L_b/64)-1, then the tree tiles (the ancestor mask of a
+// node for tree tile t is one 64-bit word).  All units' tiles are laid end to
+// end and CTA c takes the contiguous range [c*T/P, (c+1)*T/P) ("stream-K"), so
+// every SM gets the same number of tiles whatever the ragged cache lengths.
+// A unit wholly inside one CTA writes its bf16 output directly; a unit cut by
+// range boundaries writes one partial (normalised O, base-2 log-sum-exp) per
+// piece, and the CTA that completes the unit's last piece (a per-unit counter,
+// fence + atomic, no waiting) merges the pieces and writes the output.
+//
+// Roles (10 warps):
+//   warps 0-3 / 4-7   softmax of M tile 0 / 1: thread t owns row t = TMEM lane t
+//   warp 8            TMA producer: Q rows (4-D box: d x group head x node),
+//                     64-key K and V tiles into 4-stage rings (128-byte swizzle)
+//   warp 9            MMA issuer (one lane): S_m = Q_m K^T (M128 N64 K128) into a
+//                     double-buffered TMEM S_m; O_m += P_m V (M128 N128 K64)
+// TMEM: S[2][2] (4 x 64 columns) + O[2] (2 x 128 columns) = all 512 columns.
+// The online softmax keeps a lazily updated row max (O is rescaled in TMEM only
+// when the max grows by more than 2^8).  Every mbarrier wait is bounded; on a
+// timeout the CTA raises CURE_DEVERR_TIMEOUT, drains and leaves.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
@@ -28,30 +36,42 @@ namespace {
 
 using namespace tc;
 
-constexpr int BM = kAttnRowsCta;  // 128
-constexpr int BN = kAttnKeys;     // 64
+constexpr int BM = kAttnRowsCta;  // 128 rows per M tile
+constexpr int BN = kAttnKeys;     // 64 keys per tile
 constexpr int D = kAttnD;         // 128
-constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS = 0;    // S buffers: columns [0, 64) and [64, 128)
-constexpr uint32_t kColO = 128;  // O: columns [128, 256)
+constexpr int NS = 4;             // K and V ring stages
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 512;
 
 constexpr int kQHalf = BM * 64 * 2;   // 16 KiB: [128 rows][64 d]
 constexpr int kKVHalf = BN * 64 * 2;  // 8 KiB: [64 keys][64 d]
-constexpr int kTile = 2 * kKVHalf;    // one K or V tile
-constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + 2 * kQHalf;
-constexpr int kOffV = kOffK + 2 * kTile;
-constexpr int kOffP = kOffV + 2 * kTile;
-constexpr int kOffBar = kOffP + BM * BN * 2;
-enum { B_KFULL = 0, B_VFULL = 2, B_KEMPTY = 4, B_VEMPTY = 6, B_SFULL = 8, B_SFREE = 10,
-       B_PFULL = 12, B_PVDONE = 13, B_DRAIN = 14, kNumBars = 15 };
-constexpr int kOffTmemSlot = kOffBar + 8 * kNumBars;
+constexpr int kTile = 2 * kKVHalf;    // one K or V tile (16 KiB)
+constexpr int kPTile = BM * BN * 2;   // 16 KiB
+constexpr int kOffQ = 0;                          // Q[m][half]
+constexpr int kOffP = kOffQ + 4 * kQHalf;         // P[m]
+constexpr int kOffK = kOffP + 2 * kPTile;         // K[stage]
+constexpr int kOffV = kOffK + NS * kTile;         // V[stage]
+constexpr int kOffMisc = kOffV + NS * kTile;      // 229376
+enum {
+  B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + NS, B_VFULL = B_KEMPTY + NS,
+  B_VEMPTY = B_VFULL + NS, B_SFULL = B_VEMPTY + NS, B_SFREE = B_SFULL + 4, B_PFULL = B_SFREE + 4,
+  B_PVDONE = B_PFULL + 2, B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 1
+};
+constexpr int kOffTmemSlot = kOffMisc + 8 * kNumBars;
 constexpr int kOffAbort = kOffTmemSlot + 4;
-constexpr int kSmemBytes = kOffBar + 128;
-static_assert(kOffAbort + 4 <= kSmemBytes, "bookkeeping fits");
+constexpr int kOffLast = kOffAbort + 4;
+constexpr int kOffPrefix = kOffLast + 8;             // int tiles_start[B+1], units_start[B+1]
+constexpr int kSmemBytes = kOffPrefix + 8 * (kAttnMaxBatch + 1);
+static_assert(kSmemBytes <= 232448, "fits the 227 KiB opt-in");
 
+constexpr uint32_t kColS = 0;    // S[m][buf]: columns m*128 + buf*64
+constexpr uint32_t kColO = 256;  // O[m]:      columns 256 + m*128
 constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
+
+struct Bar {
+  uint32_t base;
+  __device__ __forceinline__ uint32_t operator()(int i) const { return base + 8u * (uint32_t)i; }
+};
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                              int* err, bool honour_abort) {
@@ -87,16 +107,76 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                : "memory");
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
-               "r"(valid ? 16 : 0)
-               : "memory");
+__device__ __forceinline__ void named_sync_softmax() {  // warps 0-7
+  asm volatile("bar.sync 1, 256;" ::: "memory");
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1, int c2, int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
+
+// One unit piece owned by this CTA.
+struct Seg {
+  int b, h, rg;    // unit
+  int u;           // global unit id
+  int t0, t1;      // tile range within the unit
+  int T;           // tiles of the unit
+  int nct;         // cache tiles of the unit
+  int L, n;        // cache length, tree nodes
+  int part, parts; // piece index and piece count of the unit
+  int slot;        // first workspace slot of the unit
+};
+
+struct Sched {
+  const int* tiles_start;  // smem [B+1]
+  const int* units_start;  // smem [B+1]
+  int B, Hkv, P;
+  long long Ttot;
+  const int* cache_len;
+  const int* n_nodes;
+  int cap, n_max;
+  __device__ int owner(long long g) const {  // the CTA whose range holds tile g
+    return (int)(((g + 1) * (long long)P - 1) / Ttot);
+  }
+  // The piece that starts at global tile g and ends no later than g_end.
+  __device__ Seg at(long long g, long long g_end) const {
+    int lo = 0, hi = B;  // largest b with tiles_start[b] <= g
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (tiles_start[mid] <= g) lo = mid;
+      else hi = mid;
+    }
+    Seg s;
+    s.b = lo;
+    s.L = max(0, min(cache_len[lo], cap));
+    s.n = max(1, min(n_nodes[lo], n_max));
+    s.nct = (s.L + BN - 1) / BN;
+    s.T = s.nct + (s.n + BN - 1) / BN;
+    const long long local = g - tiles_start[lo];
+    const int uib = (int)(local / s.T);
+    s.rg = uib / Hkv;
+    s.h = uib % Hkv;
+    s.u = units_start[lo] + uib;
+    s.t0 = (int)(local % s.T);
+    s.t1 = (int)min((long long)s.T, (long long)s.t0 + (g_end - g));
+    const long long ustart = g - s.t0;
+    const int o0 = owner(ustart), o1 = owner(ustart + s.T - 1);
+    s.parts = o1 - o0 + 1;
+    s.part = owner(g) - o0;
+    s.slot = s.u + o0;
+    return s;
+  }
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
 tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                    const __grid_constant__ CUtensorMap tm_tk,
-                    const __grid_constant__ CUtensorMap tm_tv, const AttnArgs A) {
+                    const __grid_constant__ CUtensorMap tm_tk, const __grid_constant__ CUtensorMap tm_tv,
+                    const __grid_constant__ CUtensorMap tm_q, const AttnArgs A) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sb = smem_u32(smem);
@@ -104,350 +184,491 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     if (tid == 0) flag(A.err, CURE_DEVERR_ALIGN);
     return;
   }
-
-  const int rb = blockIdx.x, split = blockIdx.y;
-  const int Hkv = A.kv.heads_kv;
-  const int b = blockIdx.z / Hkv, h = blockIdx.z % Hkv;
-  int L = A.cache_len[b];
-  int n = A.n_nodes[b];
-  if (L < 0 || L > A.cap || n < 1 || n > A.n_max) {
-    if (tid == 0 && rb == 0 && split == 0 && h == 0)
-      flag(A.err, (L < 0 || L > A.cap) ? CURE_DEVERR_SLOT : CURE_DEVERR_NODES);
-    L = max(0, min(L, A.cap));
-    n = max(1, min(n, A.n_max));
-  }
-  const int rows_valid = n * A.G;
-  const int r0 = rb * BM;
-  if (r0 >= rows_valid) return;
-  const int nsplit = max(1, (L + A.chunk - 1) / A.chunk);
-  if (split >= nsplit) return;
-  const int key_beg = split * A.chunk;
-  const int key_end = min(L, key_beg + A.chunk);
-  const bool has_tree = split == nsplit - 1;
-  const int n_cache_tiles = (key_end - key_beg + BN - 1) / BN;
-  const int n_tiles = n_cache_tiles + (has_tree ? (n + BN - 1) / BN : 0);
-
-  const uint32_t bar0 = sb + kOffBar;
-  auto bar = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
+  const int B = A.batch, Hkv = A.kv.heads_kv, G = A.G;
+  const int npb = BM / G;  // tree nodes per M tile
+  const Bar bar{sb + kOffMisc};
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffAbort);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(smem + kOffLast);
+  int* tiles_start = reinterpret_cast<int*>(smem + kOffPrefix);
+  int* units_start = tiles_start + (kAttnMaxBatch + 1);
 
+  // ---------------------------------------------------------------- set-up
   if (tid == 0) {
-    for (int i = 0; i < 2; ++i) {
+    mbar_init(bar(B_QFULL), 1);
+    mbar_init(bar(B_QEMPTY), 1);
+    for (int i = 0; i < NS; ++i) {
       mbar_init(bar(B_KFULL + i), 1);
-      mbar_init(bar(B_VFULL + i), 1);
       mbar_init(bar(B_KEMPTY + i), 1);
+      mbar_init(bar(B_VFULL + i), 1);
       mbar_init(bar(B_VEMPTY + i), 1);
+    }
+    for (int i = 0; i < 4; ++i) {
       mbar_init(bar(B_SFULL + i), 1);
       mbar_init(bar(B_SFREE + i), 128);
     }
-    mbar_init(bar(B_PFULL), 128);
-    mbar_init(bar(B_PVDONE), 1);
+    for (int m = 0; m < 2; ++m) {
+      mbar_init(bar(B_PFULL + m), 128);
+      mbar_init(bar(B_PVDONE + m), 1);
+      mbar_init(bar(B_OFREE + m), 128);
+    }
     mbar_init(bar(B_DRAIN), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 0) tmem_alloc(sb + kOffTmemSlot, kTmemCols);
-  if (warp == 4 && lane == 0) {
+  if (warp == 8 && lane == 0) {
+    tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
-    if (has_tree) {
-      tma_prefetch_desc(&tm_tk);
-      tma_prefetch_desc(&tm_tv);
+    tma_prefetch_desc(&tm_tk);
+    tma_prefetch_desc(&tm_tv);
+  }
+  // Q rows at or past npb * G are never written by the Q copies: zero them once
+  const int pad_rows = BM - npb * G;
+  for (int c = tid; c < 4 * pad_rows * 8; c += kThreads) {
+    const int q16 = c & 7, rr = npb * G + ((c >> 3) % pad_rows), mh = (c >> 3) / pad_rows;
+    st_shared_v4(sb + kOffQ + mh * kQHalf + rr * 128 + q16 * 16, 0u, 0u, 0u, 0u);
+  }
+  // per-sequence tiles and units, and their prefix sums (warp 9 scans)
+  if (warp == 9) {
+    int run_t = 0, run_u = 0;
+    for (int base = 0; base < B; base += 32) {
+      const int b = base + lane;
+      int tb = 0, ub = 0;
+      if (b < B) {
+        int L = A.cache_len[b], n = A.n_nodes[b];
+        if (L < 0 || L > A.cap) {
+          if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_SLOT);
+          L = max(0, min(L, A.cap));
+        }
+        if (n < 1 || n > A.n_max) {
+          if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_NODES);
+          n = max(1, min(n, A.n_max));
+        }
+        const int rg = (n + 2 * npb - 1) / (2 * npb);
+        ub = rg * Hkv;
+        tb = ub * ((L + BN - 1) / BN + (n + BN - 1) / BN);
+      }
+      int it = tb, iu = ub;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int yt = __shfl_up_sync(0xffffffffu, it, off);
+        const int yu = __shfl_up_sync(0xffffffffu, iu, off);
+        if (lane >= off) {
+          it += yt;
+          iu += yu;
+        }
+      }
+      if (b < B) {
+        tiles_start[b] = run_t + it - tb;
+        units_start[b] = run_u + iu - ub;
+      }
+      run_t += __shfl_sync(0xffffffffu, it, 31);
+      run_u += __shfl_sync(0xffffffffu, iu, 31);
+    }
+    if (lane == 0) {
+      tiles_start[B] = run_t;
+      units_start[B] = run_u;
     }
   }
-
-  // Q rows of this block into the swizzled K-major layout (zero past the valid rows)
-  for (int c = tid; c < BM * 16; c += kThreads) {
-    const int row = c >> 4, ch = c & 15, half = ch >> 3, cc = ch & 7;
-    const int r = r0 + row;
-    const bool v = r < rows_valid;
-    const int j = v ? r / A.G : 0, g = v ? r % A.G : 0;
-    const uint16_t* src =
-        v ? A.q + (((int64_t)b * A.n_max + j) * A.heads_q + h * A.G + g) * D + ch * 8 : A.q;
-    cp_async16(sb + kOffQ + half * kQHalf + row * 128 + ((cc ^ (row & 7)) << 4), src, v);
-  }
-  asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffTmemSlot);
 
-  if (warp == 4) {
-    // ------------------------------------------------------------ TMA producer
-    // One 64-key tile of K (or V) into `dst`: cache tiles come from the
-    // contiguous or paged cache, the tree tiles from this step's tree rows.
-    // Physical page ids of the split are fetched 32 tiles at a time, one tile
-    // per lane (up to 8 pages of a 64-key tile in registers), and handed to
-    // lane 0 by shuffles: no dependent global load sits in front of a copy.
+  Sched sch;
+  sch.tiles_start = tiles_start;
+  sch.units_start = units_start;
+  sch.B = B;
+  sch.Hkv = Hkv;
+  sch.Ttot = tiles_start[B];
+  // with fewer tiles than CTAs only the first Ttot CTAs take part, so that every
+  // taking part owns at least one tile and a unit's pieces are its owners
+  sch.P = (int)min((long long)gridDim.x, sch.Ttot);
+  sch.cache_len = A.cache_len;
+  sch.n_nodes = A.n_nodes;
+  sch.cap = A.cap;
+  sch.n_max = A.n_max;
+  const bool takes_part = (int)blockIdx.x < sch.P;
+  const long long g_begin = takes_part ? (long long)blockIdx.x * sch.Ttot / sch.P : 0;
+  const long long g_end = takes_part ? (long long)(blockIdx.x + 1) * sch.Ttot / sch.P : 0;
+  // M tile 1 of a piece is active when its first node is a tree node
+  auto active1 = [&](const Seg& s) { return (2 * s.rg + 1) * npb < s.n; };
+
+  if (warp == 8) {
+    // ================================================================ producer
     const int ps = A.kv.page_size;
-    const int ppt = A.kv.layout == 1 ? BN / ps : 0;  // pages per tile
-    int pg[8];
-    auto fetch_pages = [&](int window) {
-      const int j = window * 32 + lane;
-#pragma unroll
-      for (int p = 0; p < 8; ++p) {
-        pg[p] = -1;
-        if (p < ppt && j < n_cache_tiles) {
-          const int tok = key_beg + j * BN + p * ps;
-          if (tok < key_end) {
-            const int page = A.kv.block_table[(int64_t)b * A.kv.max_len + tok / ps];
-            if (page < 0 || page >= A.kv.num_pages) flag(A.err, CURE_DEVERR_PAGE);
-            else pg[p] = page;  // a missing page stays -1: its box reads zeros
-          }
+    const int ppt = A.kv.layout == 1 ? BN / ps : 0;
+    const uint32_t qbytes = (uint32_t)(npb * G * 128);
+    uint32_t qc = 0, gk = 0;  // pieces started, tiles issued (ring position)
+    uint32_t k_issued = 0, v_issued = 0;
+    bool ok = true;
+    for (long long g = g_begin; ok && g < g_end;) {
+      const Seg s = sch.at(g, g_end);
+      g += s.t1 - s.t0;
+      // Q of both M tiles once the previous piece's S products are done
+      if (!wait_warp(bar(B_QEMPTY), (qc & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
+      ++qc;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar(B_QFULL), 4 * qbytes);
+        for (int m = 0; m < 2; ++m) {
+          const int node0 = (2 * s.rg + m) * npb;
+          for (int hf = 0; hf < 2; ++hf)
+            tma_load_4d(sb + kOffQ + (2 * m + hf) * kQHalf, &tm_q, bar(B_QFULL), hf * 64, 0, s.h,
+                        s.b * A.n_max + node0);
         }
       }
-    };
-    int tile_pg[8];
-    // One 64-key tile of K (or V) into `dst`: cache tiles come from the
-    // contiguous or paged cache, the tree tiles from this step's tree rows.
-    auto load_tile = [&](int j, uint32_t dst, uint32_t fb, const CUtensorMap* cache_map,
-                         const CUtensorMap* tree_map) {
-      if (j < n_cache_tiles) {
-        const int t0 = key_beg + j * BN;
-        if (A.kv.layout == 0) {
-          const int row = b * A.kv.max_len + t0;
-          for (int hf = 0; hf < 2; ++hf) tma_load_3d(dst + hf * kKVHalf, cache_map, fb, hf * 64, h, row);
-        } else {
+      __syncwarp();
+      int pg[8];
+      for (int t = s.t0; ok && t < s.t1; ++t) {
+        // page ids of up to 32 tiles, one tile per lane, fetched together
+        if (ppt > 0 && t < s.nct && ((t - s.t0) & 31) == 0) {
+          const int tl = t + lane;
 #pragma unroll
           for (int p = 0; p < 8; ++p) {
-            if (p < ppt) {
-              for (int hf = 0; hf < 2; ++hf)
-                tma_load_3d(dst + hf * kKVHalf + p * ps * 128, cache_map, fb, hf * 64, h,
-                            tile_pg[p] * ps);
+            pg[p] = -1;
+            if (p < ppt && tl < s.nct && tl < s.t1) {
+              const int tok = tl * BN + p * ps;
+              if (tok < s.L) {
+                const int page = A.kv.block_table[(int64_t)s.b * A.kv.max_len + tok / ps];
+                if (page < 0 || page >= A.kv.num_pages) flag(A.err, CURE_DEVERR_PAGE);
+                else pg[p] = page;  // a missing page stays -1: its box reads zeros
+              }
             }
           }
         }
-      } else {
-        const int row = b * A.n_max + (j - n_cache_tiles) * BN;
-        for (int hf = 0; hf < 2; ++hf) tma_load_3d(dst + hf * kKVHalf, tree_map, fb, hf * 64, h, row);
-      }
-    };
-    int k_issued = 0, v_issued = 0;
-    for (int j = 0; j < n_tiles; ++j) {
-      const int s = j & 1;
-      const uint32_t use = (uint32_t)j >> 1;
-      if (ppt > 0 && j < n_cache_tiles) {
-        if ((j & 31) == 0) fetch_pages(j >> 5);
+        int tpg[8];
 #pragma unroll
-        for (int p = 0; p < 8; ++p) tile_pg[p] = __shfl_sync(0xffffffffu, pg[p], j & 31);
+        for (int p = 0; p < 8; ++p) tpg[p] = -1;
+        if (ppt > 0 && t < s.nct) {
+#pragma unroll
+          for (int p = 0; p < 8; ++p) tpg[p] = __shfl_sync(0xffffffffu, pg[p], (t - s.t0) & 31);
+        }
+        const int st = (int)(gk % NS);
+        const uint32_t ph = ((gk / NS) & 1u) ^ 1u;
+        // The boxes of one tile are issued by several lanes at once (one box
+        // each): a single issuing thread sustains only a few boxes per
+        // microsecond, and a paged tile is 2 * (64 / page_size) boxes.
+        auto issue = [&](uint32_t dst, uint32_t fb, const CUtensorMap* cmap, const CUtensorMap* tmap) {
+          const int hf = lane & 1, p = lane >> 1;
+          if (t < s.nct) {
+            if (A.kv.layout == 0) {
+              if (lane < 2)
+                tma_load_3d(dst + hf * kKVHalf, cmap, fb, hf * 64, s.h, s.b * A.kv.max_len + t * BN);
+            } else if (p < ppt) {
+              int pgv = tpg[0];
+#pragma unroll
+              for (int q = 1; q < 8; ++q) pgv = (q == p) ? tpg[q] : pgv;
+              tma_load_3d(dst + hf * kKVHalf + p * ps * 128, cmap, fb, hf * 64, s.h, pgv * ps);
+            }
+          } else if (lane < 2) {
+            tma_load_3d(dst + hf * kKVHalf, tmap, fb, hf * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
+          }
+        };
+        if (!wait_warp(bar(B_KEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
+        if (lane == 0) mbar_arrive_expect_tx(bar(B_KFULL + st), kTile);
+        __syncwarp();
+        issue(sb + kOffK + st * kTile, bar(B_KFULL + st), &tm_k, &tm_tk);
+        __syncwarp();
+        ++k_issued;
+        if (!wait_warp(bar(B_VEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
+        if (lane == 0) mbar_arrive_expect_tx(bar(B_VFULL + st), kTile);
+        __syncwarp();
+        issue(sb + kOffV + st * kTile, bar(B_VFULL + st), &tm_v, &tm_tv);
+        __syncwarp();
+        ++v_issued;
+        ++gk;
       }
-      // K stage s frees when S(j-2) completes, V stage s when PV(j-2) does
-      if (!wait_warp(bar(B_KEMPTY + s), (use & 1u) ^ 1u, abort_flag, A.err)) break;
-      if (lane == 0) {
-        const uint32_t dk = sb + kOffK + s * kTile;
-        mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
-        load_tile(j, dk, bar(B_KFULL + s), &tm_k, &tm_tk);
-      }
-      __syncwarp();
-      k_issued = j + 1;
-      if (!wait_warp(bar(B_VEMPTY + s), (use & 1u) ^ 1u, abort_flag, A.err)) break;
-      if (lane == 0) {
-        const uint32_t dv = sb + kOffV + s * kTile;
-        mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
-        load_tile(j, dv, bar(B_VFULL + s), &tm_v, &tm_tv);
-      }
-      __syncwarp();
-      v_issued = j + 1;
     }
     if (*abort_flag) {  // let copies in flight land before the CTA's smem goes away
-      for (int jj = max(0, k_issued - 2); jj < k_issued; ++jj)
-        wait_bounded(bar(B_KFULL + (jj & 1)), ((uint32_t)jj >> 1) & 1u, abort_flag, A.err, false);
-      for (int jj = max(0, v_issued - 2); jj < v_issued; ++jj)
-        wait_bounded(bar(B_VFULL + (jj & 1)), ((uint32_t)jj >> 1) & 1u, abort_flag, A.err, false);
+      for (uint32_t i = (k_issued > NS ? k_issued - NS : 0); i < k_issued; ++i)
+        wait_bounded(bar(B_KFULL + i % NS), (i / NS) & 1u, abort_flag, A.err, false);
+      for (uint32_t i = (v_issued > NS ? v_issued - NS : 0); i < v_issued; ++i)
+        wait_bounded(bar(B_VFULL + i % NS), (i / NS) & 1u, abort_flag, A.err, false);
+      if (qc > 0) wait_bounded(bar(B_QFULL), (qc - 1) & 1u, abort_flag, A.err, false);
     }
-  } else if (warp == 5) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 9) {
+    // ================================================================ MMA issuer
     constexpr uint32_t idS = idesc_bf16_f32(BM, BN, false);
     constexpr uint32_t idO = idesc_bf16_f32(BM, D, true);
-    auto issue_s = [&](int j) -> bool {
-      const int s = j & 1;
-      const uint32_t use = (uint32_t)j >> 1;
-      if (!wait_warp(bar(B_KFULL + s), use & 1u, abort_flag, A.err)) return false;
-      if (!wait_warp(bar(B_SFREE + s), (use & 1u) ^ 1u, abort_flag, A.err)) return false;
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t qa = sb + kOffQ, ka = sb + kOffK + s * kTile;
+    uint32_t qc = 0, gk = 0, sc[2] = {0, 0}, pc[2] = {0, 0}, oc[2] = {0, 0};
+    bool ok = true;
+    for (long long g = g_begin; ok && g < g_end;) {
+      const Seg s = sch.at(g, g_end);
+      g += s.t1 - s.t0;
+      const int nm = active1(s) ? 2 : 1;
+      const int n = s.t1 - s.t0;
+      if (!wait_warp(bar(B_QFULL), qc & 1u, abort_flag, A.err)) { ok = false; break; }
+      ++qc;
+      const uint32_t gk0 = gk;
+      auto issue_s = [&](int j) -> bool {
+        const uint32_t gt = gk0 + (uint32_t)j;
+        const int st = (int)(gt % NS);
+        if (!wait_warp(bar(B_KFULL + st), (gt / NS) & 1u, abort_flag, A.err)) return false;
+        for (int m = 0; m < nm; ++m) {
+          const int buf = (int)(sc[m] & 1u);
+          if (!wait_warp(bar(B_SFREE + 2 * m + buf), ((sc[m] >> 1) & 1u) ^ 1u, abort_flag, A.err))
+            return false;
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t qa = sb + kOffQ + 2 * m * kQHalf, ka = sb + kOffK + st * kTile;
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t oq = (ks >> 2) * kQHalf + (ks & 3) * 32;
-          const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
-          mma_bf16_ss(tmem + kColS + s * BN, sdesc_sw128(qa + oq, 16, 1024),
-                      sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
+            for (int ks = 0; ks < 8; ++ks) {
+              const uint32_t oq = (ks >> 2) * kQHalf + (ks & 3) * 32;
+              const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
+              mma_bf16_ss(tmem + kColS + m * 128 + buf * BN, sdesc_sw128(qa + oq, 16, 1024),
+                          sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
+            }
+            mma_commit(bar(B_SFULL + 2 * m + buf));
+          }
+          __syncwarp();
+          ++sc[m];
         }
-        mma_commit(bar(B_SFULL + s));
-        mma_commit(bar(B_KEMPTY + s));
-      }
-      __syncwarp();
-      return true;
-    };
-    bool ok = issue_s(0) && (n_tiles < 2 || issue_s(1));
-    for (int j = 0; ok && j < n_tiles; ++j) {
-      const int s = j & 1;
-      const uint32_t use = (uint32_t)j >> 1;
-      if (!wait_warp(bar(B_PFULL), (uint32_t)j & 1u, abort_flag, A.err)) break;
-      if (!wait_warp(bar(B_VFULL + s), use & 1u, abort_flag, A.err)) break;
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t pa = sb + kOffP, va = sb + kOffV + s * kTile;
+        if (lane == 0) {
+          mma_commit(bar(B_KEMPTY + st));
+          if (j == n - 1) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
+        }
+        __syncwarp();
+        return true;
+      };
+      ok = issue_s(0) && (n < 2 || issue_s(1));
+      for (int j = 0; ok && j < n; ++j) {
+        const uint32_t gt = gk0 + (uint32_t)j;
+        const int st = (int)(gt % NS);
+        for (int m = 0; ok && m < nm; ++m) {
+          if (!wait_warp(bar(B_PFULL + m), pc[m] & 1u, abort_flag, A.err)) { ok = false; break; }
+          if (j == 0 && !wait_warp(bar(B_OFREE + m), (oc[m] & 1u) ^ 1u, abort_flag, A.err)) {
+            ok = false;
+            break;
+          }
+          if (m == 0 && !wait_warp(bar(B_VFULL + st), (gt / NS) & 1u, abort_flag, A.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t pa = sb + kOffP + m * kPTile, va = sb + kOffV + st * kTile;
 #pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-          mma_bf16_ss(tmem + kColO, sdesc_sw128(pa + ks * 32, 16, 1024),
-                      sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
-                      (j > 0 || ks > 0) ? 1u : 0u);
+            for (int ks = 0; ks < 4; ++ks)
+              mma_bf16_ss(tmem + kColO + m * 128, sdesc_sw128(pa + ks * 32, 16, 1024),
+                          sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
+                          (j > 0 || ks > 0) ? 1u : 0u);
+            mma_commit(bar(B_PVDONE + m));
+          }
+          __syncwarp();
+          ++pc[m];
+          if (j == 0) ++oc[m];
         }
-        mma_commit(bar(B_PVDONE));
-        mma_commit(bar(B_VEMPTY + s));
+        if (!ok) break;
+        if (lane == 0) mma_commit(bar(B_VEMPTY + st));
+        __syncwarp();
+        if (j + 2 < n && !issue_s(j + 2)) { ok = false; break; }
       }
-      __syncwarp();
-      // S(j+2) reuses the S buffer that softmax(j) has finished reading
-      if (j + 2 < n_tiles && !issue_s(j + 2)) break;
+      gk = gk0 + (uint32_t)n;
     }
-    // every MMA issued by this warp has completed once the drain barrier flips
     if (lane == 0) mma_commit(bar(B_DRAIN));
     __syncwarp();
     wait_bounded(bar(B_DRAIN), 0, abort_flag, A.err, false);
   } else {
-    // ------------------------------------------------------------ softmax (rows)
-    const int row = tid;
-    const int r = r0 + row;
-    const bool vrow = r < rows_valid;
-    const int jrow = vrow ? r / A.G : 0;
-    uint64_t an[4] = {0ull, 0ull, 0ull, 0ull};
-    if (has_tree && vrow) {
-#pragma unroll
-      for (int w = 0; w < 4; ++w)
-        if (w < A.W) an[w] = A.anc[((int64_t)b * A.n_max + jrow) * A.W + w];
-    }
-    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+    // ================================================================ softmax
+    const int m = warp >> 2;   // M tile
+    const int row = tid & 127; // row within the M tile = TMEM lane
+    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float c = A.scale_log2;
-    float m_run = -INFINITY, l_run = 0.f;
+    uint32_t sc = 0, pc = 0, gk = 0;
     bool ok = true;
-    for (int j = 0; j < n_tiles; ++j) {
-      const int s = j & 1;
-      const uint32_t use = (uint32_t)j >> 1;
-      if (!wait_warp(bar(B_SFULL + s), use & 1u, abort_flag, A.err)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      uint32_t u0[32], u1[32];
-      tmem_ld32(tl + kColS + s * BN, u0);
-      tmem_ld32(tl + kColS + s * BN + 32, u1);
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(bar(B_SFREE + s));
+    for (long long g = g_begin; g < g_end;) {
+      const Seg s = sch.at(g, g_end);
+      g += s.t1 - s.t0;
+      const int n = s.t1 - s.t0;
+      const uint32_t gk0 = gk;
+      gk += (uint32_t)n;
+      const bool act = m == 0 || active1(s);
+      const int node0 = (2 * s.rg + m) * npb;
+      const int node = node0 + row / G, gh = row % G;
+      const bool vrow = act && row < npb * G && node < s.n;
+      float m_run = -INFINITY, l_run = 0.f;
+      if (act && ok) {
+        for (int jj = 0; jj < n; ++jj) {
+          const int t = s.t0 + jj;
+          const int buf = (int)(sc & 1u);
+          if (!wait_warp(bar(B_SFULL + 2 * m + buf), (sc >> 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+          tc_fence_after();
+          uint32_t u0[32], u1[32];
+          tmem_ld32(tl + kColS + m * 128 + buf * BN, u0);
+          tmem_ld32(tl + kColS + m * 128 + buf * BN + 32, u1);
+          tmem_wait_ld();
+          tc_fence_before();
+          mbar_arrive(bar(B_SFREE + 2 * m + buf));
+          ++sc;
 
-      const bool tree = j >= n_cache_tiles;
-      float x[64];
-      if (tree) {
-        const int wi = j - n_cache_tiles;
-        const uint64_t word = wi == 0 ? an[0] : wi == 1 ? an[1] : wi == 2 ? an[2] : an[3];
+          const bool tree = t >= s.nct;
+          float x[64];
+          int valid;
+          if (tree) {
+            const int wi = t - s.nct;
+            valid = min(BN, s.n - wi * BN);
+            const uint64_t word = vrow ? A.anc[((int64_t)s.b * A.n_max + node) * A.W + wi] : 0ull;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          x[i] = ((word >> i) & 1ull) ? __uint_as_float(u0[i]) * c : -INFINITY;
-          x[32 + i] = ((word >> (32 + i)) & 1ull) ? __uint_as_float(u1[i]) * c : -INFINITY;
-        }
-      } else {
-        const int lim = key_end - (key_beg + j * BN);
+            for (int i = 0; i < 32; ++i) {
+              x[i] = ((word >> i) & 1ull) ? __uint_as_float(u0[i]) * c : -INFINITY;
+              x[32 + i] = ((word >> (32 + i)) & 1ull) ? __uint_as_float(u1[i]) * c : -INFINITY;
+            }
+          } else {
+            valid = min(BN, s.L - t * BN);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          x[i] = i < lim ? __uint_as_float(u0[i]) * c : -INFINITY;
-          x[32 + i] = 32 + i < lim ? __uint_as_float(u1[i]) * c : -INFINITY;
-        }
-      }
-      float mx[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = x[i];
-#pragma unroll
-      for (int i = 8; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], x[i]);
-      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-      const float m_new = fmaxf(m_run, mt);
-      const bool need = m_new > m_run + 8.0f;
-      // the row max used for this tile's probabilities (lazily updated)
-      const float m_use = need ? m_new : m_run;
-      const float base = m_use == -INFINITY ? 0.f : m_use;
-      uint32_t pk[32];
-      float sm[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float p0 = ex2(x[2 * i] - base), p1 = ex2(x[2 * i + 1] - base);
-        sm[i & 3] += p0 + p1;
-        pk[i] = pack_bf16(p0, p1);
-      }
-
-      // P and O are free once the previous PV product has completed
-      if (j > 0) {
-        if (!wait_warp(bar(B_PVDONE), (uint32_t)(j - 1) & 1u, abort_flag, A.err)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, need)) {
-          const float alpha = need ? ex2(m_run - m_new) : 1.f;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint32_t o[32];
-            tmem_ld32(tl + kColO + q * 32, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            tmem_st32(tl + kColO + q * 32, o);
+            for (int i = 0; i < 32; ++i) {
+              x[i] = i < valid ? __uint_as_float(u0[i]) * c : -INFINITY;
+              x[32 + i] = 32 + i < valid ? __uint_as_float(u1[i]) * c : -INFINITY;
+            }
           }
-          tmem_wait_st();
-        }
-      }
-      if (need) {
-        l_run *= ex2(m_run - m_new);
-        m_run = m_new;
-      }
-      l_run += (sm[0] + sm[1]) + (sm[2] + sm[3]);
-      const uint32_t prow = sb + kOffP + row * 128;
+          float mx[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        st_shared_v4(prow + ((q ^ (row & 7)) << 4), pk[4 * q], pk[4 * q + 1], pk[4 * q + 2],
-                     pk[4 * q + 3]);
-
-      // a partial tile: zero the V rows past the last valid key so that their
-      // (unspecified) contents cannot reach O through 0 * NaN
-      const int valid = tree ? min(BN, n - (j - n_cache_tiles) * BN)
-                             : min(BN, key_end - (key_beg + j * BN));
-      if (valid < BN) {
-        if (!wait_warp(bar(B_VFULL + s), use & 1u, abort_flag, A.err)) {
-          ok = false;
-          break;
+          for (int i = 0; i < 8; ++i) mx[i] = x[i];
+#pragma unroll
+          for (int i = 8; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], x[i]);
+          const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                 fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+          const float m_new = fmaxf(m_run, mt);
+          const bool need = m_new > m_run + 8.0f;
+          const float m_use = need ? m_new : m_run;
+          const float base = m_use == -INFINITY ? 0.f : m_use;
+          uint32_t pk[32];
+          float sm[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float p0 = ex2(x[2 * i] - base), p1 = ex2(x[2 * i + 1] - base);
+            sm[i & 3] += p0 + p1;
+            pk[i] = pack_bf16(p0, p1);
+          }
+          // P_m and O_m are free once the previous PV product has completed
+          if (jj > 0) {
+            if (!wait_warp(bar(B_PVDONE + m), (pc - 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+            tc_fence_after();
+            if (__any_sync(0xffffffffu, need)) {
+              const float alpha = need ? ex2(m_run - m_new) : 1.f;
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                uint32_t o[32];
+                tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                tmem_st32(tl + kColO + m * 128 + q * 32, o);
+              }
+              tmem_wait_st();
+            }
+          }
+          if (need) {
+            l_run *= ex2(m_run - m_new);
+            m_run = m_new;
+          }
+          l_run += (sm[0] + sm[1]) + (sm[2] + sm[3]);
+          const uint32_t prow = sb + kOffP + m * kPTile + row * 128;
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            st_shared_v4(prow + ((q ^ (row & 7)) << 4), pk[4 * q], pk[4 * q + 1], pk[4 * q + 2],
+                         pk[4 * q + 3]);
+          // M tile 0 zeroes the V rows past the last valid key of a partial tile
+          // so that their unspecified contents cannot reach O through 0 * NaN
+          if (m == 0 && valid < BN) {
+            const uint32_t gt = gk0 + (uint32_t)jj;
+            const int st = (int)(gt % NS);
+            if (!wait_warp(bar(B_VFULL + st), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+            const uint32_t vb = sb + kOffV + st * kTile;
+            const int nch = (BN - valid) * 16;
+            for (int q = row; q < nch; q += BM) {
+              const int rr = valid + (q >> 4), hf = (q >> 3) & 1, cc = q & 7;
+              st_shared_v4(vb + hf * kKVHalf + rr * 128 + cc * 16, 0u, 0u, 0u, 0u);
+            }
+          }
+          fence_proxy_async_smem();
+          tc_fence_before();
+          mbar_arrive(bar(B_PFULL + m));
+          ++pc;
         }
-        const uint32_t vb = sb + kOffV + s * kTile;
-        const int nch = (BN - valid) * 16;
-        for (int q = row; q < nch; q += BM) {
-          const int rr = valid + (q >> 4), hf = (q >> 3) & 1, cc = q & 7;
-          st_shared_v4(vb + hf * kKVHalf + rr * 128 + cc * 16, 0u, 0u, 0u, 0u);
-        }
+        if (ok && !wait_warp(bar(B_PVDONE + m), (pc - 1) & 1u, abort_flag, A.err)) ok = false;
+        if (ok) tc_fence_after();
       }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(bar(B_PFULL));
-    }
-    if (ok && wait_warp(bar(B_PVDONE), (uint32_t)(n_tiles - 1) & 1u, abort_flag, A.err)) {
-      tc_fence_after();
+      // ---- epilogue of the piece
+      const bool whole = s.t0 == 0 && s.t1 == s.T;
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      const int64_t pbase = ((int64_t)blockIdx.z * A.splits + split) * A.rows_pad;
-      float* dst = A.ws_o + (pbase + r) * D;
+      const int64_t prow_idx = (int64_t)(s.slot + s.part) * (2 * BM) + m * BM + row;
+      uint16_t* orow =
+          A.out + (((int64_t)s.b * A.n_max + min(node, A.n_max - 1)) * A.heads_q + s.h * G + gh) * D;
+      if (act && ok) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint32_t o[32];
-        tmem_ld32(tl + kColO + q * 32, o);
-        tmem_wait_ld();
-        if (vrow) {
+        for (int q = 0; q < 4; ++q) {
+          uint32_t o[32];
+          tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+          tmem_wait_ld();
+          if (vrow) {
+            if (whole) {
 #pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4*>(dst + q * 32 + i) =
-                make_float4(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv,
-                            __uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
+              for (int i = 0; i < 32; i += 8) {
+                uint4 v;
+                v.x = pack_bf16(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv);
+                v.y = pack_bf16(__uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
+                v.z = pack_bf16(__uint_as_float(o[i + 4]) * inv, __uint_as_float(o[i + 5]) * inv);
+                v.w = pack_bf16(__uint_as_float(o[i + 6]) * inv, __uint_as_float(o[i + 7]) * inv);
+                *reinterpret_cast<uint4*>(orow + q * 32 + i) = v;
+              }
+            } else {
+              float* dst = A.ws_o + prow_idx * D + q * 32;
+#pragma unroll
+              for (int i = 0; i < 32; i += 4)
+                *reinterpret_cast<float4*>(dst + i) =
+                    make_float4(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv,
+                                __uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(bar(B_OFREE + m));
+      }
+      if (!whole) {
+        if (vrow && ok) A.ws_lse[prow_idx] = m_run + log2f(l_run);
+        // the CTA that completes the unit's last piece merges the pieces
+        __threadfence();
+        named_sync_softmax();
+        if (tid == 0) {
+          int last = 0;
+          if (!*abort_flag) {
+            const int old = atomicAdd(A.cnt + s.u, 1);
+            last = old == s.parts - 1;
+            if (last) A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+          }
+          *last_flag = last;
+        }
+        named_sync_softmax();
+        if (*last_flag && vrow) {
+          __threadfence();
+          const int64_t r0 = (int64_t)s.slot * (2 * BM) + m * BM + row;
+          float M = -INFINITY;
+          for (int p = 0; p < s.parts; ++p) M = fmaxf(M, __ldcg(A.ws_lse + r0 + (int64_t)p * 2 * BM));
+          float wsum = 0.f;
+          for (int p = 0; p < s.parts; ++p) wsum += ex2(__ldcg(A.ws_lse + r0 + (int64_t)p * 2 * BM) - M);
+          const float winv = 1.f / wsum;
+          for (int q = 0; q < D; q += 8) {
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            for (int p = 0; p < s.parts; ++p) {
+              const int64_t rp = r0 + (int64_t)p * 2 * BM;
+              const float w = ex2(__ldcg(A.ws_lse + rp) - M) * winv;
+              const float4 a = __ldcg(reinterpret_cast<const float4*>(A.ws_o + rp * D + q));
+              const float4 bq = __ldcg(reinterpret_cast<const float4*>(A.ws_o + rp * D + q + 4));
+              acc[0] += w * a.x; acc[1] += w * a.y; acc[2] += w * a.z; acc[3] += w * a.w;
+              acc[4] += w * bq.x; acc[5] += w * bq.y; acc[6] += w * bq.z; acc[7] += w * bq.w;
+            }
+            uint4 v;
+            v.x = pack_bf16(acc[0], acc[1]);
+            v.y = pack_bf16(acc[2], acc[3]);
+            v.z = pack_bf16(acc[4], acc[5]);
+            v.w = pack_bf16(acc[6], acc[7]);
+            *reinterpret_cast<uint4*>(orow + q) = v;
+          }
         }
       }
-      if (vrow) A.ws_lse[pbase + r] = m_run + log2f(l_run);
     }
   }
 
@@ -473,9 +694,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// [rows][Hkv][128] bf16 viewed as a 3-D tensor (d, head, row); boxes of
-// 64 d x 1 head x box_rows rows with 128-byte swizzle.
-bool make_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv, int box_rows) {
+// [rows][Hkv][128] bf16 viewed as (d, head, row); boxes of 64 d x 1 head x box_rows.
+bool make_kv_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hkv, (cuuint64_t)rows};
@@ -483,6 +703,20 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv, int box_
   cuuint32_t box[3] = {64, 1, (cuuint32_t)box_rows};
   cuuint32_t es[3] = {1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// q [tokens][Hkv][G][128] bf16 viewed as (d, group head, kv head, token); boxes
+// of 64 d x G x 1 x npb tokens: the rows of one M tile, (node, g) packed.
+bool make_q_map(CUtensorMap* m, const void* base, uint64_t tokens, int Hkv, int G, int npb) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)G, (cuuint64_t)Hkv, (cuuint64_t)tokens};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)G * D * 2, (cuuint64_t)Hkv * G * D * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)G, 1, (cuuint32_t)npb};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -502,20 +736,24 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
     attr_done.fetch_or(bit);
   }
   const int Hkv = A.kv.heads_kv;
-  CUtensorMap mk, mv, mtk, mtv;
+  CUtensorMap mk, mv, mtk, mtv, mq;
   bool ok;
   if (A.kv.layout == 0) {
     const uint64_t rows = (uint64_t)A.batch * A.kv.max_len;
-    ok = make_map(&mk, A.kc, rows, Hkv, BN) && make_map(&mv, A.vc, rows, Hkv, BN);
+    ok = make_kv_map(&mk, A.kc, rows, Hkv, BN) && make_kv_map(&mv, A.vc, rows, Hkv, BN);
   } else {
     const uint64_t rows = (uint64_t)A.kv.num_pages * A.kv.page_size;
-    ok = make_map(&mk, A.kc, rows, Hkv, A.kv.page_size) &&
-         make_map(&mv, A.vc, rows, Hkv, A.kv.page_size);
+    ok = make_kv_map(&mk, A.kc, rows, Hkv, A.kv.page_size) &&
+         make_kv_map(&mv, A.vc, rows, Hkv, A.kv.page_size);
   }
   const uint64_t trows = (uint64_t)A.batch * A.n_max;
-  ok = ok && make_map(&mtk, A.tk, trows, Hkv, BN) && make_map(&mtv, A.tv, trows, Hkv, BN);
+  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_kv_map(&mtv, A.tv, trows, Hkv, BN) &&
+       make_q_map(&mq, A.q, trows, Hkv, A.G, BM / A.G);
   if (!ok) return cudaErrorInvalidValue;
-  tree_attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(mk, mv, mtk, mtv, A);
+  // the per-unit piece counters start at zero (the kernel leaves them at zero)
+  e = cudaMemsetAsync(A.cnt, 0, sizeof(int) * (size_t)A.units_max, s);
+  if (e != cudaSuccess) return e;
+  tree_attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(mk, mv, mtk, mtv, mq, A);
   return cudaGetLastError();
 }
 

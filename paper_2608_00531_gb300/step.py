@@ -92,6 +92,6 @@ class RepairVerifyStep:
 
     @property
     def launches_per_step(self) -> int:
-        """Kernels one step launches: scan, tree, layers x (attention + reduce),
-        target argmax + walk, gather + finalize."""
-        return 1 + 1 + 2 * self.layers + 2 + 2
+        """Library kernels one step launches: scan, tree, one attention kernel per
+        layer, target argmax + walk, gather + finalize."""
+        return 1 + 1 + self.layers + 2 + 2

@@ -94,10 +94,12 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(env):
 def test_noalloc_rejects_shapes_beyond_its_scratch(env):
     lib, cure = env
     x = _inputs(3)
-    # a 16 384-page capacity per sequence at batch 4 needs far more than 64 MiB
-    big = cure.kv_desc(x["Hkv"], 128, 16384, x["table"], 16, x["npages"])
-    assert cure.cure_tree_attn_workspace_size(x["B"], x["N"], x["Hq"], big) > SCRATCH
+    # batch 200 with 28/4 heads needs more split-KV scratch than 64 MiB; the
+    # buffers are too small for that batch, but nothing may be launched
+    kv = cure.kv_desc(x["Hkv"], 128, x["table"].shape[1], x["table"], 16, x["npages"])
+    assert cure.cure_tree_attn_workspace_size(200, x["N"], x["Hq"], kv) > SCRATCH
     out = torch.zeros_like(x["q"])
-    assert _call_noalloc(lib, x, big, out) == CAPACITY
+    big = dict(x, B=200)
+    assert _call_noalloc(lib, big, kv, out) == CAPACITY
     torch.cuda.synchronize()
     assert int(out.abs().sum()) == 0      # nothing was launched
