@@ -13,18 +13,21 @@
 // piece, and the CTA that completes the unit's last piece (a per-unit counter,
 // fence + atomic, no waiting) merges the pieces and writes the output.
 //
-// Roles (10 warps):
-//   warps 0-3 / 4-7   M tile 0 / 1: thread t owns row t = TMEM lane t; it loads
-//                     its Q row into TMEM, runs the online softmax and writes
-//                     its bf16 probabilities back into TMEM
-//   warp 8            TMA producer: 64-key K and V tiles into 6-stage rings
-//                     (128-byte swizzle), page ids prefetched, boxes issued
-//                     from several lanes
-//   warp 9            MMA issuer (one lane): S_m = Q_m K^T (A = Q_m in TMEM,
-//                     M128 N64 K128); O_m += P_m V (A = P_m in TMEM, M128 N128 K64)
-// TMEM (512 columns): Q[2] (2 x 64 bf16 pairs) | S[2] (2 x 64; P_m overwrites
-// the first 32 columns of S_m) | O[2] (2 x 128).  With both A operands in TMEM
-// the tensor core reads only the 64-key K or V tile from shared memory.
+// Roles (11 warps):
+//   warps 0-3 / 4-7   softmax of M tile 0 / 1: thread t owns row t = TMEM lane t
+//                     and writes its bf16 probabilities back into TMEM
+//   warp 8            TMA producer: Q rows (4-D box: d x group head x node),
+//                     64-key K and V tiles into 4-stage rings (128-byte
+//                     swizzle), page ids prefetched, boxes issued from
+//                     several lanes
+//   warps 9 / 10      MMA issuers (one lane each) of M tile 0 / 1:
+//                     S_m = Q_m K^T (M128 N64 K128) into a double-buffered
+//                     TMEM S_m; O_m += P_m V (A = P_m in TMEM, M128 N128 K64).
+//                     Issuing a tcgen05.mma costs the issuing thread about as
+//                     long as a 64-column product takes to run, so each M
+//                     tile has its own issuer.
+// TMEM (512 columns): S[2][2] (4 x 64; P overwrites the first 32 columns of
+// its S buffer) | O[2] (2 x 128).
 // The online softmax keeps a lazily updated row max (O is rescaled in TMEM only
 // when the max grows by more than 2^8).  Every mbarrier wait is bounded; on a
 // timeout the CTA raises CURE_DEVERR_TIMEOUT, drains and leaves.
@@ -44,19 +47,21 @@ using namespace tc;
 constexpr int BM = kAttnRowsCta;  // 128 rows per M tile
 constexpr int BN = kAttnKeys;     // 64 keys per tile
 constexpr int D = kAttnD;         // 128
-constexpr int NS = 6;             // K and V ring stages
-constexpr int kThreads = 320;
+constexpr int NS = 4;             // K and V ring stages
+constexpr int kThreads = 352;     // 11 warps
 constexpr uint32_t kTmemCols = 512;
 
+constexpr int kQHalf = BM * 64 * 2;   // 16 KiB: [128 rows][64 d]
 constexpr int kKVHalf = BN * 64 * 2;  // 8 KiB: [64 keys][64 d]
 constexpr int kTile = 2 * kKVHalf;    // one K or V tile (16 KiB)
-constexpr int kOffK = 0;                          // K[stage]
+constexpr int kOffQ = 0;                          // Q[m][half]
+constexpr int kOffK = kOffQ + 4 * kQHalf;         // K[stage]
 constexpr int kOffV = kOffK + NS * kTile;         // V[stage]
 constexpr int kOffMisc = kOffV + NS * kTile;      // 196608
 enum {
-  B_KFULL = 0, B_KEMPTY = B_KFULL + NS, B_VFULL = B_KEMPTY + NS, B_VEMPTY = B_VFULL + NS,
-  B_QFULL = B_VEMPTY + NS, B_SFULL = B_QFULL + 2, B_PFULL = B_SFULL + 2, B_PVDONE = B_PFULL + 2,
-  B_OREADY = B_PVDONE + 2, B_OFREE = B_OREADY + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 1
+  B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + NS, B_VFULL = B_KEMPTY + NS,
+  B_VEMPTY = B_VFULL + NS, B_SFULL = B_VEMPTY + NS, B_PFULL = B_SFULL + 4, B_PVDONE = B_PFULL + 2,
+  B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 2
 };
 constexpr int kOffTmemSlot = kOffMisc + 8 * kNumBars;
 constexpr int kOffAbort = kOffTmemSlot + 4;
@@ -65,9 +70,8 @@ constexpr int kOffPrefix = kOffLast + 8;             // int tiles_start[B+1], un
 constexpr int kSmemBytes = kOffPrefix + 8 * (kAttnMaxBatch + 1);
 static_assert(kSmemBytes <= 232448, "fits the 227 KiB opt-in");
 
-constexpr uint32_t kColQ = 0;    // Q[m]: columns m*64 .. m*64+63 (bf16 pairs)
-constexpr uint32_t kColS = 128;  // S[m]: columns 128 + m*64; P[m] in its first 32
-constexpr uint32_t kColO = 256;  // O[m]: columns 256 + m*128
+constexpr uint32_t kColS = 0;    // S[m][buf]: columns m*128 + buf*64; P in the first 32
+constexpr uint32_t kColO = 256;  // O[m]:      columns 256 + m*128
 constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
 struct Bar {
@@ -111,6 +115,15 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 
 __device__ __forceinline__ void named_sync_softmax() {  // warps 0-7
   asm volatile("bar.sync 1, 256;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1, int c2, int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
 }
 
 // One unit piece owned by this CTA.
@@ -169,7 +182,7 @@ struct Sched {
 __global__ void __launch_bounds__(kThreads, 1)
 tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                     const __grid_constant__ CUtensorMap tm_tk, const __grid_constant__ CUtensorMap tm_tv,
-                    const AttnArgs A) {
+                    const __grid_constant__ CUtensorMap tm_q, const AttnArgs A) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sb = smem_u32(smem);
@@ -187,30 +200,37 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
 
   // ---------------------------------------------------------------- set-up
   if (tid == 0) {
+    mbar_init(bar(B_QFULL), 1);
+    mbar_init(bar(B_QEMPTY), 2);
     for (int i = 0; i < NS; ++i) {
       mbar_init(bar(B_KFULL + i), 1);
-      mbar_init(bar(B_KEMPTY + i), 1);
+      mbar_init(bar(B_KEMPTY + i), 2);
       mbar_init(bar(B_VFULL + i), 1);
-      mbar_init(bar(B_VEMPTY + i), 1);
+      mbar_init(bar(B_VEMPTY + i), 2);
     }
+    for (int i = 0; i < 4; ++i) mbar_init(bar(B_SFULL + i), 1);  // [m][buf]
     for (int m = 0; m < 2; ++m) {
-      mbar_init(bar(B_QFULL + m), 128);
-      mbar_init(bar(B_SFULL + m), 1);
       mbar_init(bar(B_PFULL + m), 128);
       mbar_init(bar(B_PVDONE + m), 1);
-      mbar_init(bar(B_OREADY + m), 1);
       mbar_init(bar(B_OFREE + m), 128);
+      mbar_init(bar(B_DRAIN + m), 1);
     }
-    mbar_init(bar(B_DRAIN), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   if (warp == 0) tmem_alloc(sb + kOffTmemSlot, kTmemCols);
   if (warp == 8 && lane == 0) {
+    tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
     tma_prefetch_desc(&tm_tk);
     tma_prefetch_desc(&tm_tv);
+  }
+  // Q rows at or past npb * G are never written by the Q copies: zero them once
+  const int pad_rows = BM - npb * G;
+  for (int c = tid; c < 4 * pad_rows * 8; c += kThreads) {
+    const int q16 = c & 7, rr = npb * G + ((c >> 3) % pad_rows), mh = (c >> 3) / pad_rows;
+    st_shared_v4(sb + kOffQ + mh * kQHalf + rr * 128 + q16 * 16, 0u, 0u, 0u, 0u);
   }
   // per-sequence tiles and units, and their prefix sums (warp 9 scans)
   if (warp == 9) {
@@ -254,6 +274,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       units_start[B] = run_u;
     }
   }
+  fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -282,12 +303,26 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     // ================================================================ producer
     const int ps = A.kv.page_size;
     const int ppt = A.kv.layout == 1 ? BN / ps : 0;
-    uint32_t gk = 0;  // tiles issued (ring position)
+    const uint32_t qbytes = (uint32_t)(npb * G * 128);
+    uint32_t qc = 0, gk = 0;  // pieces started, tiles issued (ring position)
     uint32_t k_issued = 0, v_issued = 0;
     bool ok = true;
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
       g += s.t1 - s.t0;
+      // Q of both M tiles once the previous piece's S products are done
+      if (!wait_warp(bar(B_QEMPTY), (qc & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
+      ++qc;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar(B_QFULL), 4 * qbytes);
+        for (int m = 0; m < 2; ++m) {
+          const int node0 = (2 * s.rg + m) * npb;
+          for (int hf = 0; hf < 2; ++hf)
+            tma_load_4d(sb + kOffQ + (2 * m + hf) * kQHalf, &tm_q, bar(B_QFULL), hf * 64, 0, s.h,
+                        s.b * A.n_max + node0);
+        }
+      }
+      __syncwarp();
       int pg[8];
       for (int t = s.t0; ok && t < s.t1; ++t) {
         // page ids of up to 32 tiles, one tile per lane, fetched together
@@ -354,108 +389,109 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         wait_bounded(bar(B_KFULL + i % NS), (i / NS) & 1u, abort_flag, A.err, false);
       for (uint32_t i = (v_issued > NS ? v_issued - NS : 0); i < v_issued; ++i)
         wait_bounded(bar(B_VFULL + i % NS), (i / NS) & 1u, abort_flag, A.err, false);
+      if (qc > 0) wait_bounded(bar(B_QFULL), (qc - 1) & 1u, abort_flag, A.err, false);
     }
-  } else if (warp == 9) {
-    // ================================================================ MMA issuer
+  } else if (warp >= 9) {
+    // ================================================================ MMA issuers
+    // warp 9 + m issues the products of M tile m
+    const int m = warp - 9;
     constexpr uint32_t idS = idesc_bf16_f32(BM, BN, false);
     constexpr uint32_t idO = idesc_bf16_f32(BM, D, true);
-    uint32_t gk = 0, qc[2] = {0, 0}, pc[2] = {0, 0}, oc[2] = {0, 0};
+    uint32_t qc = 0, gk = 0, sc = 0, pvw = 0, pc = 0, oc = 0;
     bool ok = true;
-    // S_m(j) = Q_m K(j)^T; the caller has checked that K(j) is resident
-    auto issue_s = [&](int m, uint32_t gt) {
-      const uint32_t ka = sb + kOffK + (gt % NS) * kTile;
-      if (lane == 0) {
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
-          mma_bf16_ts(tmem + kColS + m * 64, tmem + kColQ + m * 64 + ks * 8,
-                      sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
-        }
-        mma_commit(bar(B_SFULL + m));
-      }
-      __syncwarp();
-    };
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
       g += s.t1 - s.t0;
-      const int nm = active1(s) ? 2 : 1;
       const int n = s.t1 - s.t0;
       const uint32_t gk0 = gk;
-      for (int m = 0; ok && m < nm; ++m) {
-        if (!wait_warp(bar(B_QFULL + m), qc[m] & 1u, abort_flag, A.err)) ok = false;
-        ++qc[m];
+      gk += (uint32_t)n;
+      if (!wait_warp(bar(B_QFULL), qc & 1u, abort_flag, A.err)) { ok = false; break; }
+      ++qc;
+      if (!(m == 0 || active1(s))) {
+        // an M tile without rows in this piece still releases every stage
+        for (int j = 0; ok && j < n; ++j) {
+          const uint32_t gt = gk0 + (uint32_t)j;
+          if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+          if (lane == 0) mbar_arrive(bar(B_KEMPTY + gt % NS));
+          if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+          if (lane == 0) mbar_arrive(bar(B_VEMPTY + gt % NS));
+          __syncwarp();
+        }
+        if (lane == 0) mbar_arrive(bar(B_QEMPTY));
+        __syncwarp();
+        continue;
       }
-      if (!ok) break;
-      if (!wait_warp(bar(B_KFULL + gk0 % NS), (gk0 / NS) & 1u, abort_flag, A.err)) break;
-      tc_fence_after();
-      for (int m = 0; m < nm; ++m) issue_s(m, gk0);
-      if (lane == 0) mma_commit(bar(B_KEMPTY + gk0 % NS));
-      __syncwarp();
+      // S #sc goes to buffer sc & 1, whose previous S / P (#sc - 2) must have
+      // been consumed by its PV product
+      // (PV completions are consumed in order, each before a later one can have
+      // happened: an mbarrier parity wait two phases late would block)
+      auto issue_s = [&](uint32_t gt, bool last_s) -> bool {
+        while (pvw + 2 <= sc) {
+          if (!wait_warp(bar(B_PVDONE + m), pvw & 1u, abort_flag, A.err)) return false;
+          ++pvw;
+        }
+        if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) return false;
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t qa = sb + kOffQ + 2 * m * kQHalf, ka = sb + kOffK + (gt % NS) * kTile;
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t oq = (ks >> 2) * kQHalf + (ks & 3) * 32;
+            const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
+            mma_bf16_ss(tmem + kColS + m * 128 + (sc & 1u) * BN, sdesc_sw128(qa + oq, 16, 1024),
+                        sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
+          }
+          mma_commit(bar(B_SFULL + 2 * m + (sc & 1u)));
+          mma_commit(bar(B_KEMPTY + gt % NS));
+          if (last_s) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
+        }
+        __syncwarp();
+        ++sc;
+        return true;
+      };
+      ok = issue_s(gk0, n == 1) && (n < 2 || issue_s(gk0 + 1, n == 2));
       for (int j = 0; ok && j < n; ++j) {
         const uint32_t gt = gk0 + (uint32_t)j;
-        const int st = (int)(gt % NS);
-        for (int m = 0; ok && m < nm; ++m) {
-          if (!wait_warp(bar(B_PFULL + m), pc[m] & 1u, abort_flag, A.err)) { ok = false; break; }
-          if (j == 0 && !wait_warp(bar(B_OFREE + m), (oc[m] & 1u) ^ 1u, abort_flag, A.err)) {
-            ok = false;
-            break;
-          }
-          if (m == 0 && !wait_warp(bar(B_VFULL + st), (gt / NS) & 1u, abort_flag, A.err)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          if (lane == 0) {
-            const uint32_t va = sb + kOffV + st * kTile;
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-              mma_bf16_ts(tmem + kColO + m * 128, tmem + kColS + m * 64 + ks * 8,
-                          sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
-                          (j > 0 || ks > 0) ? 1u : 0u);
-            mma_commit(bar(B_PVDONE + m));
-            if (j == n - 1) mma_commit(bar(B_OREADY + m));
-          }
-          __syncwarp();
-          ++pc[m];
-          if (j == 0) ++oc[m];
+        if (!wait_warp(bar(B_PFULL + m), pc & 1u, abort_flag, A.err)) { ok = false; break; }
+        if (j == 0) {
+          if (!wait_warp(bar(B_OFREE + m), (oc & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
+          ++oc;
+        }
+        if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+        // every earlier PV has completed (the softmax saw PV #pc-1 finish
+        // before it published P #pc): consume those completions first
+        while (ok && pvw < pc) {
+          if (!wait_warp(bar(B_PVDONE + m), pvw & 1u, abort_flag, A.err)) ok = false;
+          ++pvw;
         }
         if (!ok) break;
-        if (lane == 0) mma_commit(bar(B_VEMPTY + st));
-        __syncwarp();
-        if (j + 1 < n) {
-          // S_m(j+1) overwrites the columns that PV_m(j) reads P_m(j) from: wait
-          // for that product, then issue (the other M tile's work is queued)
-          if (!wait_warp(bar(B_KFULL + (gt + 1) % NS), ((gt + 1) / NS) & 1u, abort_flag, A.err)) {
-            ok = false;
-            break;
-          }
-          for (int m = 0; ok && m < nm; ++m) {
-            if (!wait_warp(bar(B_PVDONE + m), (pc[m] - 1) & 1u, abort_flag, A.err)) { ok = false; break; }
-            tc_fence_after();
-            issue_s(m, gt + 1);
-          }
-          if (!ok) break;
-          if (lane == 0) mma_commit(bar(B_KEMPTY + (gt + 1) % NS));
-          __syncwarp();
-        } else {
-          // the last product of the piece: consume the PV completions so that
-          // their phases stay in step with the waits above
-          for (int m = 0; ok && m < nm; ++m)
-            if (!wait_warp(bar(B_PVDONE + m), (pc[m] - 1) & 1u, abort_flag, A.err)) ok = false;
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t va = sb + kOffV + (gt % NS) * kTile;
+          const uint32_t pa = tmem + kColS + m * 128 + (pc & 1u) * BN;  // P over S's columns
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16_ts(tmem + kColO + m * 128, pa + ks * 8,
+                        sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
+                        (j > 0 || ks > 0) ? 1u : 0u);
+          mma_commit(bar(B_PVDONE + m));
+          mma_commit(bar(B_VEMPTY + gt % NS));
         }
+        __syncwarp();
+        ++pc;
+        if (j + 2 < n && !issue_s(gt + 2, j + 2 == n - 1)) { ok = false; break; }
       }
-      gk = gk0 + (uint32_t)n;
     }
-    if (lane == 0) mma_commit(bar(B_DRAIN));
+    if (lane == 0) mma_commit(bar(B_DRAIN + m));
     __syncwarp();
-    wait_bounded(bar(B_DRAIN), 0, abort_flag, A.err, false);
+    wait_bounded(bar(B_DRAIN + m), 0, abort_flag, A.err, false);
   } else {
     // ================================================================ softmax
     const int m = warp >> 2;   // M tile
     const int row = tid & 127; // row within the M tile = TMEM lane
     const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float c = A.scale_log2;
-    uint32_t sc = 0, oc = 0, gk = 0;
+    uint32_t sc = 0, pvc = 0, gk = 0;
     bool ok = true;
     for (long long g = g_begin; g < g_end;) {
       const Seg s = sch.at(g, g_end);
@@ -469,36 +505,17 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       const bool vrow = act && row < npb * G && node < s.n;
       float m_run = -INFINITY, l_run = 0.f;
       if (act && ok) {
-        // this row's query into TMEM (the previous piece's S products, which
-        // read Q_m, have all completed: their results were consumed)
-        {
-          const uint4* qsrc = reinterpret_cast<const uint4*>(
-              A.q + (((int64_t)s.b * A.n_max + (vrow ? node : 0)) * A.heads_q + s.h * G + gh) * D);
-#pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            uint32_t qv[32];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              uint4 v = vrow ? __ldg(qsrc + half * 8 + i) : make_uint4(0u, 0u, 0u, 0u);
-              qv[4 * i] = v.x;
-              qv[4 * i + 1] = v.y;
-              qv[4 * i + 2] = v.z;
-              qv[4 * i + 3] = v.w;
-            }
-            tmem_st32(tl + kColQ + m * 64 + half * 32, qv);
-          }
-          tmem_wait_st();
-          tc_fence_before();
-          mbar_arrive(bar(B_QFULL + m));
-        }
         for (int jj = 0; jj < n; ++jj) {
           const int t = s.t0 + jj;
-          if (!wait_warp(bar(B_SFULL + m), sc & 1u, abort_flag, A.err)) { ok = false; break; }
+          // one barrier per S buffer: a buffer is refilled only after the PV of
+          // its previous tile, so it never runs two phases ahead of this wait
+          const uint32_t buf = sc & 1u;
+          if (!wait_warp(bar(B_SFULL + 2 * m + buf), (sc >> 1) & 1u, abort_flag, A.err)) { ok = false; break; }
           ++sc;
           tc_fence_after();
           uint32_t u0[32], u1[32];
-          tmem_ld32(tl + kColS + m * 64, u0);
-          tmem_ld32(tl + kColS + m * 64 + 32, u1);
+          tmem_ld32(tl + kColS + m * 128 + buf * BN, u0);
+          tmem_ld32(tl + kColS + m * 128 + buf * BN + 32, u1);
           tmem_wait_ld();
 
           const bool tree = t >= s.nct;
@@ -540,20 +557,25 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             sm[i & 3] += p0 + p1;
             pk[i] = pack_bf16(p0, p1);
           }
-          // P_m(j) over the first 32 columns of S_m.  S_m(j) completing means the
-          // products issued before it, PV_m(j-1) included, have completed, so
-          // O_m is stable for the rescale below.
-          tmem_st32(tl + kColS + m * 64, pk);
-          if (jj > 0 && __any_sync(0xffffffffu, need)) {
-            const float alpha = need ? ex2(m_run - m_new) : 1.f;
+          // P over the first 32 columns of this tile's S buffer (its previous P
+          // was consumed before this S was computed into it)
+          tmem_st32(tl + kColS + m * 128 + buf * BN, pk);
+          // O_m is stable once the previous PV product has completed
+          if (jj > 0) {
+            if (!wait_warp(bar(B_PVDONE + m), pvc & 1u, abort_flag, A.err)) { ok = false; break; }
+            ++pvc;
+            tc_fence_after();
+            if (__any_sync(0xffffffffu, need)) {
+              const float alpha = need ? ex2(m_run - m_new) : 1.f;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              uint32_t o[32];
-              tmem_ld32(tl + kColO + m * 128 + q * 32, o);
-              tmem_wait_ld();
+              for (int q = 0; q < 4; ++q) {
+                uint32_t o[32];
+                tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+                tmem_wait_ld();
 #pragma unroll
-              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-              tmem_st32(tl + kColO + m * 128 + q * 32, o);
+                for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                tmem_st32(tl + kColO + m * 128 + q * 32, o);
+              }
             }
           }
           if (need) {
@@ -561,9 +583,10 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             m_run = m_new;
           }
           l_run += (sm[0] + sm[1]) + (sm[2] + sm[3]);
-          // M tile 0 zeroes the V rows past the last valid key of a partial tile
-          // so that their unspecified contents cannot reach O through 0 * NaN
-          if (m == 0 && valid < BN) {
+          // the V rows past the last valid key of a partial tile are zeroed (by
+          // both M tiles: the second writes the same zeros) so that their
+          // unspecified contents cannot reach O through 0 * NaN
+          if (valid < BN) {
             const uint32_t gt = gk0 + (uint32_t)jj;
             const int st = (int)(gt % NS);
             if (!wait_warp(bar(B_VFULL + st), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
@@ -579,8 +602,10 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           tc_fence_before();
           mbar_arrive(bar(B_PFULL + m));
         }
-        if (ok && !wait_warp(bar(B_OREADY + m), oc & 1u, abort_flag, A.err)) ok = false;
-        ++oc;
+        if (ok) {
+          if (!wait_warp(bar(B_PVDONE + m), pvc & 1u, abort_flag, A.err)) ok = false;
+          ++pvc;
+        }
         if (ok) tc_fence_after();
       }
       // ---- epilogue of the piece
@@ -699,6 +724,20 @@ bool make_kv_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv, int b
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// q [tokens][Hkv][G][128] bf16 viewed as (d, group head, kv head, token); boxes
+// of 64 d x G x 1 x npb tokens: the rows of one M tile, (node, g) packed.
+bool make_q_map(CUtensorMap* m, const void* base, uint64_t tokens, int Hkv, int G, int npb) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)G, (cuuint64_t)Hkv, (cuuint64_t)tokens};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)G * D * 2, (cuuint64_t)Hkv * G * D * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)G, 1, (cuuint32_t)npb};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
@@ -714,7 +753,7 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
     attr_done.fetch_or(bit);
   }
   const int Hkv = A.kv.heads_kv;
-  CUtensorMap mk, mv, mtk, mtv;
+  CUtensorMap mk, mv, mtk, mtv, mq;
   bool ok;
   if (A.kv.layout == 0) {
     const uint64_t rows = (uint64_t)A.batch * A.kv.max_len;
@@ -725,12 +764,13 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
          make_kv_map(&mv, A.vc, rows, Hkv, A.kv.page_size);
   }
   const uint64_t trows = (uint64_t)A.batch * A.n_max;
-  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_kv_map(&mtv, A.tv, trows, Hkv, BN);
+  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_kv_map(&mtv, A.tv, trows, Hkv, BN) &&
+       make_q_map(&mq, A.q, trows, Hkv, A.G, BM / A.G);
   if (!ok) return cudaErrorInvalidValue;
   // the per-unit piece counters start at zero (the kernel leaves them at zero)
   e = cudaMemsetAsync(A.cnt, 0, sizeof(int) * (size_t)A.units_max, s);
   if (e != cudaSuccess) return e;
-  tree_attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(mk, mv, mtk, mtv, A);
+  tree_attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(mk, mv, mtk, mtv, mq, A);
   return cudaGetLastError();
 }
 
