@@ -101,12 +101,33 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# ------------------------------------------------------------------ ranks
+def rank_seed(base_seed: int, rank: int) -> int:
+    """Each rank draws its own batch (weak scaling: the per-GPU work is fixed)."""
+    return base_seed + 7 * rank
+
+
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The job's time is the slowest rank's; every rank gets it."""
+    if world == 1:
+        return ms
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_steps_per_s(ms_max: float, steps: int, world: int) -> float:
+    """Whole-job throughput: the steps all ranks ran over the slowest rank's time."""
+    return world * steps / (ms_max / 1e3)
+
+
 # ------------------------------------------------------------------ workload
 def make_workload(dev, rank: int, layers_override=None):
     from paper_2608_00531_gb300 import cure, workload as W
     from paper_2608_00531_gb300.step import RepairVerifyStep, StepInputs
     w = W.WORKLOADS[WORKLOAD]
-    seed = w.seed + 7 * rank
+    seed = rank_seed(w.seed, rank)
     layers = layers_override or w.layers
     B, K, N, D = w.batch, w.block, w.n_max, 128
     d = W.draft_block(w, seed=seed)
@@ -318,12 +339,9 @@ def main():
     t1.record(stream)
     torch.cuda.synchronize()
     clocks = clk.stop()
-    ms = t0.elapsed_time(t1)
+    ms = max_over_ranks(t0.elapsed_time(t1), world, dev)
     if world > 1:
         import torch.distributed as dist
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
         dist.barrier()
     assert cure.cure_device_error() == 0
     attn_ms = [ev_attn[s][2 * l].elapsed_time(ev_attn[s][2 * l + 1]) for s in range(args.steps) for l in range(Ly)]
@@ -334,13 +352,13 @@ def main():
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(wl, st, kcs, vcs, dev, max(3, min(args.steps, 10)))
+        e2e = run_e2e(wl, st, kcs, vcs, dev, max(3, min(args.steps, 10)), world)
 
     if rank != 0:
         return
     pk = peaks()
     ms_step = ms / args.steps
-    value = world * args.steps / (ms / 1e3)
+    value = job_steps_per_s(ms, args.steps, world)
     attn_gbs = alg["attn_bytes"] / (attn_avg * 1e-3) / 1e9
     attn_tflops = alg["attn_flops"] / (attn_avg * 1e-3) / 1e12
     scan_gbs = alg["scan_bytes"] / (scan_avg * 1e-3) / 1e9
@@ -382,10 +400,10 @@ def main():
     print(json.dumps(out), flush=True)
 
 
-def run_e2e(wl, st, kcs, vcs, dev, steps):
+def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
     """Same step through the public API with inputs in pinned host memory:
     host-to-device copies of the step's inputs and a device-to-host read of
-    the accept results inside the timed region."""
+    the accept results inside the timed region.  Whole-job value over ranks."""
     from paper_2608_00531_gb300.step import StepInputs
     x = wl["x"]
     host = {k_: getattr(x, k_).cpu().pin_memory() for k_ in ("draft_logits", "root_tok", "cache_len", "q",
@@ -411,6 +429,9 @@ def run_e2e(wl, st, kcs, vcs, dev, steps):
     for _ in range(2):
         one()
     torch.cuda.synchronize()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     a.record(stream)
@@ -418,8 +439,8 @@ def run_e2e(wl, st, kcs, vcs, dev, steps):
         one()
     b.record(stream)
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b) / steps
-    return {"value": round(1e3 / ms, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
+    ms = max_over_ranks(a.elapsed_time(b), world, dev) / steps
+    return {"value": round(job_steps_per_s(ms * steps, steps, world), 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 4), "steps": steps}
 
 
