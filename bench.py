@@ -32,8 +32,20 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
+# DRAM bytes (read + write) of one tree-attention launch on this workload, from
+# one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
+# source with the given sha256 prefix; another source reports null
+ATTN_TRAFFIC = {"4a9788da06d0f806": 315_496_448}
+
 METRIC = "repair-verify steps/s at batch 32, block 16; tree-attn & vocab-scan HBM GB/s vs peak"
 WORKLOAD = "serve32"
+
+
+def attn_source_digest() -> str:
+    import hashlib
+    src = os.path.join(ROOT, "paper_2608_00531_gb300", "csrc", "k_attn_tc.cu")
+    with open(src, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
 def peaks():
@@ -49,15 +61,23 @@ def peaks():
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while the timed
+    region runs; samples are time-stamped on arrival and only those taken
+    between `mark_start` and `mark_stop` are summarised."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    INTERVAL_MS = 50
 
     def __init__(self, dev_index: int):
         self.proc = None
         self.dev_index = dev_index
+        self.lines = []
+        self.t0 = self.t1 = None
+        self.thread = None
 
-    def start(self):
+    def start(self, wait_first_s: float = 5.0):
+        import threading
         try:
             bus = None
             try:
@@ -65,24 +85,47 @@ class ClockSampler:
                 bus = "%08X:%02X:%02X.0" % (pr.pci_domain_id, pr.pci_bus_id, pr.pci_device_id)
             except Exception:
                 bus = None
-            cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-lms", "200"]
+            cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                   "-lms", str(self.INTERVAL_MS)]
             if bus:
                 cmd += ["--id=" + bus]
             self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
+            return
+
+        def reader():
+            for line in self.proc.stdout:
+                self.lines.append((time.time(), line))
+
+        self.thread = threading.Thread(target=reader, daemon=True)
+        self.thread.start()
+        t_end = time.time() + wait_first_s   # the first sample shows the sampler is live
+        while not self.lines and time.time() < t_end and self.proc.poll() is None:
+            time.sleep(0.01)
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_stop(self):
+        self.t1 = time.time()
 
     def stop(self):
         if self.proc is None:
             return None
+        time.sleep(2 * self.INTERVAL_MS / 1e3)
         self.proc.terminate()
         try:
-            out, _ = self.proc.communicate(timeout=5)
+            self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-            out, _ = self.proc.communicate()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+        t0 = self.t0 if self.t0 is not None else 0.0
+        t1 = self.t1 if self.t1 is not None else time.time()
+        inside = [ln for ts, ln in self.lines if t0 <= ts <= t1 + self.INTERVAL_MS / 1e3]
         sm, mx, reasons = [], [], set()
-        for line in out.strip().splitlines():
+        for line in inside:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
@@ -98,7 +141,7 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "interval_ms": self.INTERVAL_MS}
 
 
 # ------------------------------------------------------------------ ranks
@@ -262,7 +305,7 @@ def cpu_baseline(budget_s: float = 12.0):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -326,18 +369,20 @@ def main():
                             cache_len_out=st.cache_len_out, out=st.rs)
 
     clk = ClockSampler(local)
+    clk.start()
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
-    clk.start()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    clk.mark_start()
     t0.record(stream)
     for s in range(args.steps):
         timed_step(s)
     t1.record(stream)
     torch.cuda.synchronize()
+    clk.mark_stop()
     clocks = clk.stop()
     ms = max_over_ranks(t0.elapsed_time(t1), world, dev)
     if world > 1:
@@ -371,7 +416,10 @@ def main():
     else:
         roof = {"bound": "tensor", "achieved": round(attn_tflops, 1), "peak": pk["bf16_tflops_sustained"],
                 "unit": "TFLOP/s", "frac": round(attn_tflops / pk["bf16_tflops_sustained"], 4)}
-    roof.update({"traffic": None, "kernel": "tree attention (tree_attn_tc_kernel, persistent, split units merged in-kernel), per layer",
+    roof.update({"traffic": ATTN_TRAFFIC.get(attn_source_digest()),
+                 "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of this kernel source "
+                                   "(one layer of this workload); null when the source has changed",
+                 "kernel": "tree attention (tree_attn_tc_kernel, persistent, split units merged in-kernel), per layer",
                  "algorithmic_bytes_per_launch": alg["attn_bytes"],
                  "algorithmic_flops_per_launch": alg["attn_flops"], "avg_launch_ms": round(attn_avg, 4),
                  "peak_source": pk["source"] + " (MEASURED_PEAKS.json hbm_gbs)"})
