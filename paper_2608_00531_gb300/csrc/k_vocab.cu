@@ -1,13 +1,18 @@
 // Stage 1 (Sec. 3.3, Eq. 2) and the target argmax of stage 5 (Sec. 3.5, greedy
 // decoding): one streaming pass over bf16 vocabulary rows.
 //
-// Each row is split over a thread-block cluster of S CTAs.  Every thread
-// streams 16-byte vectors (8 bf16 logits) with non-allocating loads and keeps
-// a register top-k list ordered by (value desc, id asc) and, for stage 1, an
-// online base-2 log-sum-exp (running max + rescaled sum).  Lists and sums are
-// merged by warp shuffles, then across the warps of the CTA through shared
-// memory, then across the cluster through distributed shared memory by the
-// CTA of rank 0, which writes the row's result.  No global scratch is used.
+// A row is scanned by one CTA, or split over a thread-block cluster of S CTAs
+// when there are too few rows to fill the GPU.  Every thread streams 16-byte
+// vectors (8 bf16 logits) with non-allocating loads, the next vectors loaded
+// while the current ones are consumed, and keeps a register top-k list
+// ordered by (value desc, id asc) and, for stage 1, an online base-2
+// log-sum-exp (running max + rescaled sum).  A logit enters a list only if it
+// reaches the warp's threshold: the largest k-th best value over the lanes,
+// below which nothing can be in the row's top k (one lane already holds k
+// values at or above it).  Lists and sums are merged by warp shuffles, then
+// across the warps of the CTA through shared memory, then across the cluster
+// through distributed shared memory by the CTA of rank 0, which writes the
+// row's result.  No global scratch is used.
 #include <cooperative_groups.h>
 #include <float.h>
 #include <limits.h>
@@ -21,7 +26,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 2;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -114,7 +119,7 @@ struct Part {
 };
 
 template <int KT, bool LSE>
-__device__ __forceinline__ void consume8(const uint4& r, int idx, TopK<KT>& tk, Lse2& ls) {
+__device__ __forceinline__ void consume8(const uint4& r, int idx, TopK<KT>& tk, Lse2& ls, float thr) {
   float x[8];
   x[0] = bf16_lo(r.x); x[1] = bf16_hi(r.x);
   x[2] = bf16_lo(r.y); x[3] = bf16_hi(r.y);
@@ -130,13 +135,17 @@ __device__ __forceinline__ void consume8(const uint4& r, int idx, TopK<KT>& tk, 
       ls.mb = nb;
     }
     if (ls.m != -INFINITY) {
+      float e2[4];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) ls.s += ex2(fmaf(x[e], kLog2e, -ls.mb));
+      for (int e = 0; e < 4; ++e)
+        e2[e] = ex2(fmaf(x[e], kLog2e, -ls.mb)) + ex2(fmaf(x[e + 4], kLog2e, -ls.mb));
+      ls.s += (e2[0] + e2[1]) + (e2[2] + e2[3]);
     }
   }
-  if (gm >= tk.v[KT - 1]) {
+  if (gm >= thr) {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) tk.insert(x[e], idx + e);
+    for (int e = 0; e < 8; ++e)
+      if (x[e] >= thr) tk.insert(x[e], idx + e);
   }
 }
 
@@ -194,18 +203,35 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     consume1<KT, LSE>(bf16_lo(rowp[tail0 + tid]), tail0 + tid, tk, ls);
 
   const uint4* vp = reinterpret_cast<const uint4*>(rowp + a0);
-  for (int base = vb + tid; base < ve; base += kUnroll * kThreads) {
-    uint4 r[kUnroll];
+  // the trip count is uniform over the warp, so that every lane takes part in
+  // the threshold exchange
+  const int lane = tid & 31;
+  const int wb0 = vb + (tid & ~31);
+  uint4 r[kUnroll];
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    const int vi = wb0 + lane + u * kThreads;
+    if (vi < ve) r[u] = ld_stream(vp + vi);
+  }
+  float thr = tk.v[KT - 1];
+  for (int wb = wb0; wb < ve; wb += kUnroll * kThreads) {
+    uint4 nx[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int vi = base + u * kThreads;
-      if (vi < ve) r[u] = ld_stream(vp + vi);
+      const int vi = wb + lane + (kUnroll + u) * kThreads;
+      if (vi < ve) nx[u] = ld_stream(vp + vi);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int vi = base + u * kThreads;
-      if (vi < ve) consume8<KT, LSE>(r[u], a0 + (vi << 3), tk, ls);
+      const int vi = wb + lane + u * kThreads;
+      if (vi < ve) consume8<KT, LSE>(r[u], a0 + (vi << 3), tk, ls, thr);
     }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) r[u] = nx[u];
+    float th = tk.v[KT - 1];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) th = fmaxf(th, __shfl_xor_sync(0xffffffffu, th, off));
+    thr = th;
   }
 
   // ---- warp merge
@@ -222,7 +248,7 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   // ---- CTA merge
   __shared__ Part<KT, LSE> warp_part[kWarps];
   __shared__ Part<KT, LSE> cta_part;
-  const int warp = tid >> 5, lane = tid & 31;
+  const int warp = tid >> 5;
   if (lane == 0) {
 #pragma unroll
     for (int k = 0; k < KT; ++k) {
@@ -305,11 +331,14 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   }
 }
 
+// One CTA per row once the rows alone give every SM two CTAs (merging a
+// split row costs more than it gains there); else split rows over a cluster
+// of up to 8 CTAs, keeping at least two vectors per thread in each.
 int pick_split(int64_t rows, int vocab) {
   const int nvec = vocab / 8;
-  int s = (int)((16LL * num_sms() + rows - 1) / rows);
+  if (rows >= 2LL * num_sms()) return 1;
+  int s = (int)((4LL * num_sms() + rows - 1) / rows);
   s = max(1, min(s, 8));
-  // keep at least two vectors per thread in each CTA
   while (s > 1 && nvec / s < 2 * kThreads) --s;
   return s;
 }
