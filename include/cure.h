@@ -140,7 +140,9 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
  * (this step's target keys/values of the tree tokens); k_cache, v_cache: one
  * layer in the layout of `kv` (a HOST pointer).  Accumulation is float32; the
  * probabilities are rounded to bf16 before the PV product.  D = 128,
- * heads_q % heads_kv == 0, all tensor base pointers 16-byte aligned.
+ * heads_q % heads_kv == 0, scale > 0 and finite (1/sqrt(D) in the paper's
+ * models; otherwise CURE_ERR_INVALID_ARG), all tensor base pointers 16-byte
+ * aligned.
  * workspace: device scratch of at least cure_tree_attn_workspace_size() bytes,
  * 256-byte aligned (split-KV partial results).
  */

@@ -19,7 +19,7 @@ struct AttnArgs {
   int units_max;   // piece counters in the workspace
   float scale_log2;
   int* cnt;        // [units_max] pieces of each unit merged so far (zero between launches)
-  float* ws_o;     // [(units_max + kAttnMaxCtas) * 256][128] partial outputs
+  float* ws_o;     // [units_max + kAttnMaxCtas][32][256] float4 partial outputs
   float* ws_lse;   // [(units_max + kAttnMaxCtas) * 256] partial base-2 log-sum-exps
   uint16_t* out;
   int* err;

@@ -1,5 +1,6 @@
 // The C ABI (include/cure.h): host-side argument checks, then the launches.
 // Nothing here allocates device memory.
+#include <float.h>
 #include <mutex>
 
 #include "common.cuh"
@@ -144,7 +145,8 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
                            void* workspace, size_t workspace_bytes, void* stream) {
   cure_status why;
   if (!kv_ok(kv, &why)) return why;
-  if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
+  if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0 ||
+      !(scale > 0.f && scale <= FLT_MAX))
     return CURE_ERR_INVALID_ARG;
   if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
     return CURE_ERR_UNSUPPORTED;

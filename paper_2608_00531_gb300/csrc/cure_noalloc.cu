@@ -14,6 +14,7 @@
 // host code `g_attn_scratch` is only a host-side stand-in for the symbol, not
 // a device address, so its device address is looked up once per device with
 // cudaGetSymbolAddress and that address is what the kernels receive.
+#include <float.h>
 #include <mutex>
 
 #include "common.cuh"
@@ -65,7 +66,8 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
   if (kv->layout == 1 && kv->page_size != 8 && kv->page_size != 16 && kv->page_size != 32 &&
       kv->page_size != 64)
     return CURE_ERR_UNSUPPORTED;
-  if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0)
+  if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0 ||
+      !(scale > 0.f && scale <= FLT_MAX))
     return CURE_ERR_INVALID_ARG;
   if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
     return CURE_ERR_UNSUPPORTED;

@@ -3,7 +3,8 @@
 //
 // Workspace layout (caller-owned, 256-byte aligned):
 //   cnt     int32 [units_max], 256-byte rounded   pieces merged per unit
-//   ws_o    fp32  [(units_max + kAttnMaxCtas) * 256][128]   partial outputs
+//   ws_o    fp32  [units_max + kAttnMaxCtas][32][256] float4: per piece slot, column-major
+//                 partial outputs (float4 column c of row r at [slot][c][r])
 //   ws_lse  fp32  [(units_max + kAttnMaxCtas) * 256]        partial log-sum-exps
 // A unit is (sequence, kv head, row group of 2 x floor(128 / G) tree nodes);
 // a unit split across CTAs needs one slot per piece, and the pieces of all

@@ -21,13 +21,18 @@
 //                     swizzle), page ids prefetched, boxes issued from
 //                     several lanes
 //   warps 9 / 10      MMA issuers (one lane each) of M tile 0 / 1:
-//                     S_m = Q_m K^T (M128 N64 K128) into a double-buffered
-//                     TMEM S_m; O_m += P_m V (A = P_m in TMEM, M128 N128 K64).
+//                     S_m = Q_m K^T (M128 N64 K128) into TMEM S_m;
+//                     O_m += P_m V (A = P_m in TMEM, M128 N128 K64).
 //                     Issuing a tcgen05.mma costs the issuing thread about as
 //                     long as a 64-column product takes to run, so each M
 //                     tile has its own issuer.
-// TMEM (512 columns): S[2][2] (4 x 64; P overwrites the first 32 columns of
-// its S buffer) | O[2] (2 x 128).
+// TMEM (512 columns): S[2] (2 x 64) | P[2][2] (4 x 32, bf16 pairs) | O[2]
+// (2 x 128).  The softmax releases S_m as soon as it has loaded it, so the
+// next tile's S product runs while this tile's exponentials are computed; P
+// is double-buffered so that it can be written while the previous PV product
+// still reads the other buffer.  The order of one issuer is
+//   S(0), S(1), PV(0), S(2), PV(1), ...
+// and a K/V ring stage is released when the PV product of its tile is done.
 // The online softmax keeps a lazily updated row max (O is rescaled in TMEM only
 // when the max grows by more than 2^8).  Every mbarrier wait is bounded; on a
 // timeout the CTA raises CURE_DEVERR_TIMEOUT, drains and leaves.
@@ -59,8 +64,8 @@ constexpr int kOffK = kOffQ + 4 * kQHalf;         // K[stage]
 constexpr int kOffV = kOffK + NS * kTile;         // V[stage]
 constexpr int kOffMisc = kOffV + NS * kTile;      // 196608
 enum {
-  B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_KEMPTY = B_KFULL + NS, B_VFULL = B_KEMPTY + NS,
-  B_VEMPTY = B_VFULL + NS, B_SFULL = B_VEMPTY + NS, B_PFULL = B_SFULL + 4, B_PVDONE = B_PFULL + 2,
+  B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_VFULL = B_KFULL + NS, B_KVEMPTY = B_VFULL + NS,
+  B_SFULL = B_KVEMPTY + NS, B_SFREE = B_SFULL + 2, B_PFULL = B_SFREE + 2, B_PVDONE = B_PFULL + 2,
   B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 2
 };
 constexpr int kOffTmemSlot = kOffMisc + 8 * kNumBars;
@@ -70,7 +75,8 @@ constexpr int kOffPrefix = kOffLast + 8;             // int tiles_start[B+1], un
 constexpr int kSmemBytes = kOffPrefix + 8 * (kAttnMaxBatch + 1);
 static_assert(kSmemBytes <= 232448, "fits the 227 KiB opt-in");
 
-constexpr uint32_t kColS = 0;    // S[m][buf]: columns m*128 + buf*64; P in the first 32
+constexpr uint32_t kColS = 0;    // S[m]:      columns m*64
+constexpr uint32_t kColP = 128;  // P[m][buf]: columns 128 + m*64 + buf*32
 constexpr uint32_t kColO = 256;  // O[m]:      columns 256 + m*128
 constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
@@ -99,6 +105,13 @@ __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatil
                                           int* err) {
   const bool ok = wait_bounded(bar, parity, abort_flag, err, true);
   return __all_sync(0xffffffffu, ok);
+}
+
+// max of three (sm_100 and later have a three-input float max)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -204,12 +217,12 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     mbar_init(bar(B_QEMPTY), 2);
     for (int i = 0; i < NS; ++i) {
       mbar_init(bar(B_KFULL + i), 1);
-      mbar_init(bar(B_KEMPTY + i), 2);
       mbar_init(bar(B_VFULL + i), 1);
-      mbar_init(bar(B_VEMPTY + i), 2);
+      mbar_init(bar(B_KVEMPTY + i), 2);
     }
-    for (int i = 0; i < 4; ++i) mbar_init(bar(B_SFULL + i), 1);  // [m][buf]
     for (int m = 0; m < 2; ++m) {
+      mbar_init(bar(B_SFULL + m), 1);
+      mbar_init(bar(B_SFREE + m), 128);
       mbar_init(bar(B_PFULL + m), 128);
       mbar_init(bar(B_PVDONE + m), 1);
       mbar_init(bar(B_OFREE + m), 128);
@@ -310,19 +323,24 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
       g += s.t1 - s.t0;
-      // Q of both M tiles once the previous piece's S products are done
-      if (!wait_warp(bar(B_QEMPTY), (qc & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
-      ++qc;
-      if (lane == 0) {
-        mbar_arrive_expect_tx(bar(B_QFULL), 4 * qbytes);
-        for (int m = 0; m < 2; ++m) {
-          const int node0 = (2 * s.rg + m) * npb;
-          for (int hf = 0; hf < 2; ++hf)
-            tma_load_4d(sb + kOffQ + (2 * m + hf) * kQHalf, &tm_q, bar(B_QFULL), hf * 64, 0, s.h,
-                        s.b * A.n_max + node0);
+      // Q of both M tiles once the previous piece's S products are done; it
+      // is requested after the piece's first K/V tile, whose ring stage frees
+      // up independently, so that the ring refills across the piece boundary
+      auto load_q = [&]() -> bool {
+        if (!wait_warp(bar(B_QEMPTY), (qc & 1u) ^ 1u, abort_flag, A.err)) return false;
+        ++qc;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(B_QFULL), 4 * qbytes);
+          for (int m = 0; m < 2; ++m) {
+            const int node0 = (2 * s.rg + m) * npb;
+            for (int hf = 0; hf < 2; ++hf)
+              tma_load_4d(sb + kOffQ + (2 * m + hf) * kQHalf, &tm_q, bar(B_QFULL), hf * 64, 0, s.h,
+                          s.b * A.n_max + node0);
+          }
         }
-      }
-      __syncwarp();
+        __syncwarp();
+        return true;
+      };
       int pg[8];
       for (int t = s.t0; ok && t < s.t1; ++t) {
         // page ids of up to 32 tiles, one tile per lane, fetched together
@@ -369,19 +387,19 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             tma_load_3d(dst + hf * kKVHalf, tmap, fb, hf * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
           }
         };
-        if (!wait_warp(bar(B_KEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
+        if (!wait_warp(bar(B_KVEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
         if (lane == 0) mbar_arrive_expect_tx(bar(B_KFULL + st), kTile);
         __syncwarp();
         issue(sb + kOffK + st * kTile, bar(B_KFULL + st), &tm_k, &tm_tk);
         __syncwarp();
         ++k_issued;
-        if (!wait_warp(bar(B_VEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
         if (lane == 0) mbar_arrive_expect_tx(bar(B_VFULL + st), kTile);
         __syncwarp();
         issue(sb + kOffV + st * kTile, bar(B_VFULL + st), &tm_v, &tm_tv);
         __syncwarp();
         ++v_issued;
         ++gk;
+        if (t == s.t0 && !load_q()) { ok = false; break; }
       }
     }
     if (*abort_flag) {  // let copies in flight land before the CTA's smem goes away
@@ -397,7 +415,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     const int m = warp - 9;
     constexpr uint32_t idS = idesc_bf16_f32(BM, BN, false);
     constexpr uint32_t idO = idesc_bf16_f32(BM, D, true);
-    uint32_t qc = 0, gk = 0, sc = 0, pvw = 0, pc = 0, oc = 0;
+    uint32_t qc = 0, gk = 0, sc = 0, pc = 0, oc = 0;
     bool ok = true;
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
@@ -409,28 +427,47 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       ++qc;
       if (!(m == 0 || active1(s))) {
         // an M tile without rows in this piece still releases every stage
+        // (after its copy was issued, so at most once per phase)
         for (int j = 0; ok && j < n; ++j) {
           const uint32_t gt = gk0 + (uint32_t)j;
           if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
-          if (lane == 0) mbar_arrive(bar(B_KEMPTY + gt % NS));
-          if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
-          if (lane == 0) mbar_arrive(bar(B_VEMPTY + gt % NS));
+          if (lane == 0) mbar_arrive(bar(B_KVEMPTY + gt % NS));
           __syncwarp();
         }
         if (lane == 0) mbar_arrive(bar(B_QEMPTY));
         __syncwarp();
         continue;
       }
-      // S #sc goes to buffer sc & 1, whose previous S / P (#sc - 2) must have
-      // been consumed by its PV product
-      // (PV completions are consumed in order, each before a later one can have
-      // happened: an mbarrier parity wait two phases late would block)
-      auto issue_s = [&](uint32_t gt, bool last_s) -> bool {
-        while (pvw + 2 <= sc) {
-          if (!wait_warp(bar(B_PVDONE + m), pvw & 1u, abort_flag, A.err)) return false;
-          ++pvw;
+      // PV of tile jp of this piece: P #pc from its buffer, V from the ring
+      auto issue_pv = [&](int jp) -> bool {
+        const uint32_t gt = gk0 + (uint32_t)jp;
+        if (!wait_warp(bar(B_PFULL + m), pc & 1u, abort_flag, A.err)) return false;
+        if (jp == 0) {  // O_m holds the previous piece until its epilogue has read it
+          if (!wait_warp(bar(B_OFREE + m), (oc & 1u) ^ 1u, abort_flag, A.err)) return false;
+          ++oc;
         }
-        if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) return false;
+        if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) return false;
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t va = sb + kOffV + (gt % NS) * kTile;
+          const uint32_t pa = tmem + kColP + m * 64 + (pc & 1u) * 32;
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16_ts(tmem + kColO + m * 128, pa + ks * 8,
+                        sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
+                        (jp > 0 || ks > 0) ? 1u : 0u);
+          mma_commit(bar(B_PVDONE + m));
+          mma_commit(bar(B_KVEMPTY + gt % NS));  // the tile's K and V are both consumed
+        }
+        __syncwarp();
+        ++pc;
+        return true;
+      };
+      for (int j = 0; ok && j < n; ++j) {
+        const uint32_t gt = gk0 + (uint32_t)j;
+        // S_m is rewritten once the softmax has loaded the previous S
+        if (sc > 0 && !wait_warp(bar(B_SFREE + m), (sc - 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+        if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
         tc_fence_after();
         if (lane == 0) {
           const uint32_t qa = sb + kOffQ + 2 * m * kQHalf, ka = sb + kOffK + (gt % NS) * kTile;
@@ -438,49 +475,17 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           for (int ks = 0; ks < 8; ++ks) {
             const uint32_t oq = (ks >> 2) * kQHalf + (ks & 3) * 32;
             const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
-            mma_bf16_ss(tmem + kColS + m * 128 + (sc & 1u) * BN, sdesc_sw128(qa + oq, 16, 1024),
+            mma_bf16_ss(tmem + kColS + m * 64, sdesc_sw128(qa + oq, 16, 1024),
                         sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
           }
-          mma_commit(bar(B_SFULL + 2 * m + (sc & 1u)));
-          mma_commit(bar(B_KEMPTY + gt % NS));
-          if (last_s) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
+          mma_commit(bar(B_SFULL + m));
+          if (j == n - 1) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
         }
         __syncwarp();
         ++sc;
-        return true;
-      };
-      ok = issue_s(gk0, n == 1) && (n < 2 || issue_s(gk0 + 1, n == 2));
-      for (int j = 0; ok && j < n; ++j) {
-        const uint32_t gt = gk0 + (uint32_t)j;
-        if (!wait_warp(bar(B_PFULL + m), pc & 1u, abort_flag, A.err)) { ok = false; break; }
-        if (j == 0) {
-          if (!wait_warp(bar(B_OFREE + m), (oc & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
-          ++oc;
-        }
-        if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
-        // every earlier PV has completed (the softmax saw PV #pc-1 finish
-        // before it published P #pc): consume those completions first
-        while (ok && pvw < pc) {
-          if (!wait_warp(bar(B_PVDONE + m), pvw & 1u, abort_flag, A.err)) ok = false;
-          ++pvw;
-        }
-        if (!ok) break;
-        tc_fence_after();
-        if (lane == 0) {
-          const uint32_t va = sb + kOffV + (gt % NS) * kTile;
-          const uint32_t pa = tmem + kColS + m * 128 + (pc & 1u) * BN;  // P over S's columns
-#pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            mma_bf16_ts(tmem + kColO + m * 128, pa + ks * 8,
-                        sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
-                        (j > 0 || ks > 0) ? 1u : 0u);
-          mma_commit(bar(B_PVDONE + m));
-          mma_commit(bar(B_VEMPTY + gt % NS));
-        }
-        __syncwarp();
-        ++pc;
-        if (j + 2 < n && !issue_s(gt + 2, j + 2 == n - 1)) { ok = false; break; }
+        if (j > 0 && !issue_pv(j - 1)) { ok = false; break; }
       }
+      if (ok && !issue_pv(n - 1)) ok = false;
     }
     if (lane == 0) mma_commit(bar(B_DRAIN + m));
     __syncwarp();
@@ -507,59 +512,69 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       if (act && ok) {
         for (int jj = 0; jj < n; ++jj) {
           const int t = s.t0 + jj;
-          // one barrier per S buffer: a buffer is refilled only after the PV of
-          // its previous tile, so it never runs two phases ahead of this wait
-          const uint32_t buf = sc & 1u;
-          if (!wait_warp(bar(B_SFULL + 2 * m + buf), (sc >> 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+          if (!wait_warp(bar(B_SFULL + m), sc & 1u, abort_flag, A.err)) { ok = false; break; }
+          const uint32_t pbuf = sc & 1u;
           ++sc;
           tc_fence_after();
           uint32_t u0[32], u1[32];
-          tmem_ld32(tl + kColS + m * 128 + buf * BN, u0);
-          tmem_ld32(tl + kColS + m * 128 + buf * BN + 32, u1);
+          tmem_ld32(tl + kColS + m * 64, u0);
+          tmem_ld32(tl + kColS + m * 64 + 32, u1);
           tmem_wait_ld();
+          tc_fence_before();
+          mbar_arrive(bar(B_SFREE + m));  // S_m may be overwritten by the next product
 
+          // raw scores, -inf where masked; the scale is applied in the exponent
           const bool tree = t >= s.nct;
+          const int valid = tree ? min(BN, s.n - (t - s.nct) * BN) : min(BN, s.L - t * BN);
           float x[64];
-          int valid;
           if (tree) {
             const int wi = t - s.nct;
-            valid = min(BN, s.n - wi * BN);
             const uint64_t word = vrow ? A.anc[((int64_t)s.b * A.n_max + node) * A.W + wi] : 0ull;
+            const uint32_t w0 = (uint32_t)word, w1 = (uint32_t)(word >> 32);
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              x[i] = ((word >> i) & 1ull) ? __uint_as_float(u0[i]) * c : -INFINITY;
-              x[32 + i] = ((word >> (32 + i)) & 1ull) ? __uint_as_float(u1[i]) * c : -INFINITY;
+              x[i] = ((w0 >> i) & 1u) ? __uint_as_float(u0[i]) : -INFINITY;
+              x[32 + i] = ((w1 >> i) & 1u) ? __uint_as_float(u1[i]) : -INFINITY;
+            }
+          } else if (valid == BN) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              x[i] = __uint_as_float(u0[i]);
+              x[32 + i] = __uint_as_float(u1[i]);
             }
           } else {
-            valid = min(BN, s.L - t * BN);
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              x[i] = i < valid ? __uint_as_float(u0[i]) * c : -INFINITY;
-              x[32 + i] = 32 + i < valid ? __uint_as_float(u1[i]) * c : -INFINITY;
+              x[i] = i < valid ? __uint_as_float(u0[i]) : -INFINITY;
+              x[32 + i] = 32 + i < valid ? __uint_as_float(u1[i]) : -INFINITY;
             }
           }
           float mx[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) mx[i] = x[i];
+          for (int i = 0; i < 8; ++i) mx[i] = fmax3(x[i], x[8 + i], x[16 + i]);
 #pragma unroll
-          for (int i = 8; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], x[i]);
-          const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                                 fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+          for (int i = 0; i < 8; ++i) mx[i] = fmax3(mx[i], x[24 + i], x[32 + i]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) mx[i] = fmax3(mx[i], x[40 + i], x[48 + i]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], x[56 + i]);
+          const float mt = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]),
+                                 fmaxf(mx[6], mx[7])) * c;
           const float m_new = fmaxf(m_run, mt);
           const bool need = m_new > m_run + 8.0f;
           const float m_use = need ? m_new : m_run;
-          const float base = m_use == -INFINITY ? 0.f : m_use;
+          const float nbase = m_use == -INFINITY ? 0.f : -m_use;
           uint32_t pk[32];
           float sm[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float p0 = ex2(x[2 * i] - base), p1 = ex2(x[2 * i + 1] - base);
+            const float p0 = ex2(fmaf(x[2 * i], c, nbase)), p1 = ex2(fmaf(x[2 * i + 1], c, nbase));
             sm[i & 3] += p0 + p1;
             pk[i] = pack_bf16(p0, p1);
           }
-          // P over the first 32 columns of this tile's S buffer (its previous P
-          // was consumed before this S was computed into it)
-          tmem_st32(tl + kColS + m * 128 + buf * BN, pk);
+          // P #sc into its buffer: the PV product that last read it (#sc - 2)
+          // completed before the previous tile's P was published
+          tmem_st32(tl + kColP + m * 64 + pbuf * 32, pk);
           // O_m is stable once the previous PV product has completed
           if (jj > 0) {
             if (!wait_warp(bar(B_PVDONE + m), pvc & 1u, abort_flag, A.err)) { ok = false; break; }
@@ -611,7 +626,10 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       // ---- epilogue of the piece
       const bool whole = s.t0 == 0 && s.t1 == s.T;
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      const int64_t prow_idx = (int64_t)(s.slot + s.part) * (2 * BM) + m * BM + row;
+      // a piece's partial: fp32 float4 columns [32][256 rows], so that the 32
+      // rows of a warp touch 512 contiguous bytes at every column
+      const int prow = m * BM + row;
+      float4* pslot = reinterpret_cast<float4*>(A.ws_o) + (int64_t)(s.slot + s.part) * (32 * 2 * BM);
       uint16_t* orow =
           A.out + (((int64_t)s.b * A.n_max + min(node, A.n_max - 1)) * A.heads_q + s.h * G + gh) * D;
       if (act && ok) {
@@ -632,12 +650,11 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
                 *reinterpret_cast<uint4*>(orow + q * 32 + i) = v;
               }
             } else {
-              float* dst = A.ws_o + prow_idx * D + q * 32;
 #pragma unroll
-              for (int i = 0; i < 32; i += 4)
-                *reinterpret_cast<float4*>(dst + i) =
-                    make_float4(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv,
-                                __uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
+              for (int i = 0; i < 8; ++i)
+                pslot[(q * 8 + i) * (2 * BM) + prow] =
+                    make_float4(__uint_as_float(o[4 * i]) * inv, __uint_as_float(o[4 * i + 1]) * inv,
+                                __uint_as_float(o[4 * i + 2]) * inv, __uint_as_float(o[4 * i + 3]) * inv);
             }
           }
         }
@@ -645,7 +662,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         mbar_arrive(bar(B_OFREE + m));
       }
       if (!whole) {
-        if (vrow && ok) A.ws_lse[prow_idx] = m_run + log2f(l_run);
+        if (vrow && ok) A.ws_lse[(int64_t)(s.slot + s.part) * (2 * BM) + prow] = m_run + log2f(l_run);
         // the CTA that completes the unit's last piece merges the pieces
         __threadfence();
         named_sync_softmax();
@@ -661,28 +678,53 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         named_sync_softmax();
         if (*last_flag && vrow) {
           __threadfence();
-          const int64_t r0 = (int64_t)s.slot * (2 * BM) + m * BM + row;
+          // O = sum_p w_p O_p with w_p = 2^(lse_p - M) / sum_q 2^(lse_q - M).
+          // Loads are batched (two pieces x eight float4 columns per thread)
+          // so that L2 latency is paid a few times per row, not per column.
+          const float* lse0 = A.ws_lse + (int64_t)s.slot * (2 * BM) + prow;
           float M = -INFINITY;
-          for (int p = 0; p < s.parts; ++p) M = fmaxf(M, __ldcg(A.ws_lse + r0 + (int64_t)p * 2 * BM));
+          for (int p = 0; p < s.parts; ++p) M = fmaxf(M, __ldcg(lse0 + (int64_t)p * 2 * BM));
           float wsum = 0.f;
-          for (int p = 0; p < s.parts; ++p) wsum += ex2(__ldcg(A.ws_lse + r0 + (int64_t)p * 2 * BM) - M);
+          for (int p = 0; p < s.parts; ++p) wsum += ex2(__ldcg(lse0 + (int64_t)p * 2 * BM) - M);
           const float winv = 1.f / wsum;
-          for (int q = 0; q < D; q += 8) {
-            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            for (int p = 0; p < s.parts; ++p) {
-              const int64_t rp = r0 + (int64_t)p * 2 * BM;
-              const float w = ex2(__ldcg(A.ws_lse + rp) - M) * winv;
-              const float4 a = __ldcg(reinterpret_cast<const float4*>(A.ws_o + rp * D + q));
-              const float4 bq = __ldcg(reinterpret_cast<const float4*>(A.ws_o + rp * D + q + 4));
-              acc[0] += w * a.x; acc[1] += w * a.y; acc[2] += w * a.z; acc[3] += w * a.w;
-              acc[4] += w * bq.x; acc[5] += w * bq.y; acc[6] += w * bq.z; acc[7] += w * bq.w;
+          const float4* base = reinterpret_cast<const float4*>(A.ws_o) + (int64_t)s.slot * (32 * 2 * BM) + prow;
+#pragma unroll 1
+          for (int c0 = 0; c0 < 32; c0 += 8) {
+            float4 acc[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+            for (int p0 = 0; p0 < s.parts; p0 += 2) {
+              const bool two = p0 + 1 < s.parts;
+              float4 va[8], vb[8];
+              const float4* pa = base + (int64_t)p0 * (32 * 2 * BM) + c0 * (2 * BM);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) va[i] = __ldcg(pa + i * (2 * BM));
+              if (two) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) vb[i] = __ldcg(pa + 32 * 2 * BM + i * (2 * BM));
+              }
+              const float wa = ex2(__ldcg(lse0 + (int64_t)p0 * 2 * BM) - M) * winv;
+              const float wb = two ? ex2(__ldcg(lse0 + (int64_t)(p0 + 1) * 2 * BM) - M) * winv : 0.f;
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                acc[i].x += wa * va[i].x; acc[i].y += wa * va[i].y;
+                acc[i].z += wa * va[i].z; acc[i].w += wa * va[i].w;
+                if (two) {
+                  acc[i].x += wb * vb[i].x; acc[i].y += wb * vb[i].y;
+                  acc[i].z += wb * vb[i].z; acc[i].w += wb * vb[i].w;
+                }
+              }
             }
-            uint4 v;
-            v.x = pack_bf16(acc[0], acc[1]);
-            v.y = pack_bf16(acc[2], acc[3]);
-            v.z = pack_bf16(acc[4], acc[5]);
-            v.w = pack_bf16(acc[6], acc[7]);
-            *reinterpret_cast<uint4*>(orow + q) = v;
+#pragma unroll
+            for (int i = 0; i < 8; i += 2) {
+              uint4 v;
+              v.x = pack_bf16(acc[i].x, acc[i].y);
+              v.y = pack_bf16(acc[i].z, acc[i].w);
+              v.z = pack_bf16(acc[i + 1].x, acc[i + 1].y);
+              v.w = pack_bf16(acc[i + 1].z, acc[i + 1].w);
+              *reinterpret_cast<uint4*>(orow + (c0 + i) * 4) = v;
+            }
           }
         }
       }
