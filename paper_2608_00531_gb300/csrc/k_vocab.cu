@@ -17,6 +17,8 @@
 #include <float.h>
 #include <limits.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace cg = cooperative_groups;
@@ -24,7 +26,7 @@ namespace cg = cooperative_groups;
 namespace cure {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 128;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 2;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -118,35 +120,60 @@ struct Part {
   float mb, s;
 };
 
-template <int KT, bool LSE>
-__device__ __forceinline__ void consume8(const uint4& r, int idx, TopK<KT>& tk, Lse2& ls, float thr) {
-  float x[8];
-  x[0] = bf16_lo(r.x); x[1] = bf16_hi(r.x);
-  x[2] = bf16_lo(r.y); x[3] = bf16_hi(r.y);
-  x[4] = bf16_lo(r.z); x[5] = bf16_hi(r.z);
-  x[6] = bf16_lo(r.w); x[7] = bf16_hi(r.w);
-  const float gm = fmaxf(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])),
-                         fmaxf(fmaxf(x[4], x[5]), fmaxf(x[6], x[7])));
-  if constexpr (LSE) {
-    if (gm > ls.m) {
-      const float nb = gm * kLog2e;
-      ls.s *= ex2(ls.mb - nb);
-      ls.m = gm;
-      ls.mb = nb;
-    }
-    if (ls.m != -INFINITY) {
-      float e2[4];
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Pairs of floats in one 64-bit register pair, for the packed f32x2
+// arithmetic of sm_100 and later (two lanes of work per instruction).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
-      for (int e = 0; e < 4; ++e)
-        e2[e] = ex2(fmaf(x[e], kLog2e, -ls.mb)) + ex2(fmaf(x[e + 4], kLog2e, -ls.mb));
-      ls.s += (e2[0] + e2[1]) + (e2[2] + e2[3]);
-    }
-  }
-  if (gm >= thr) {
+  for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+  return v;
+}
+
+// A lower bound on the warp's k-th best value, the same in every lane: the
+// largest lane-local k-th best (that lane holds k values at or above it) and
+// the k-th largest of the lane maxima (k lanes each hold one value at or
+// above it; a lane that ties the current maximum drops out with it, which can
+// only lower the bound).
+template <int KT>
+__device__ __forceinline__ float warp_kth(const TopK<KT>& tk) {
+  float t = warp_max(tk.v[KT - 1]);
+  float m = tk.v[0];
 #pragma unroll
-    for (int e = 0; e < 8; ++e)
-      if (x[e] >= thr) tk.insert(x[e], idx + e);
+  for (int k = 0; k < KT; ++k) {
+    const float mk = warp_max(m);
+    if (k == KT - 1) t = fmaxf(t, mk);
+    if (m == mk) m = -INFINITY;
   }
+  return t;
 }
 
 template <int KT, bool LSE>
@@ -203,8 +230,16 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     consume1<KT, LSE>(bf16_lo(rowp[tail0 + tid]), tail0 + tid, tk, ls);
 
   const uint4* vp = reinterpret_cast<const uint4*>(rowp + a0);
-  // the trip count is uniform over the warp, so that every lane takes part in
-  // the threshold exchange
+  // The trip count is uniform over the warp: the threshold and the log-sum-exp
+  // base are warp-wide values that all lanes take part in.
+  //  - thr: the k-th best value over the warp's lists.  A logit below it
+  //    cannot be in the row's top k (the warp already holds k values at or
+  //    above it), so lists change only in the rare steps with a logit at or
+  //    above it, after which thr is recomputed.
+  //  - mbw: base-2 exponent base of the lane sums s0 + s1 (sum of
+  //    2^(x log2e - mbw)); raised, with the sums rescaled, only when some lane
+  //    sees a logit more than 2^8 above it, so the sums stay below 2^8 per
+  //    term and the rescale is rare and uniform.
   const int lane = tid & 31;
   const int wb0 = vb + (tid & ~31);
   uint4 r[kUnroll];
@@ -213,26 +248,106 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     const int vi = wb0 + lane + u * kThreads;
     if (vi < ve) r[u] = ld_stream(vp + vi);
   }
-  float thr = tk.v[KT - 1];
-  for (int wb = wb0; wb < ve; wb += kUnroll * kThreads) {
+  float thr = warp_kth(tk);
+  float mbw = -INFINITY;
+  uint64_t sacc = f2_pack(0.f, 0.f);  // two lane sums, as one f32x2 pair
+  // one step: kUnroll vectors per lane; FULL when every lane's vectors are in
+  // range (all but a warp's last step), so that no per-vector check is needed
+  auto step = [&](int wb, auto full_tag) {
+    constexpr bool FULL = decltype(full_tag)::value;
     uint4 nx[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
       const int vi = wb + lane + (kUnroll + u) * kThreads;
       if (vi < ve) nx[u] = ld_stream(vp + vi);
     }
+    uint64_t xp[kUnroll][4];  // (lo, hi) logit pairs of each 32-bit word
+    float gmv[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int vi = wb + lane + u * kThreads;
-      if (vi < ve) consume8<KT, LSE>(r[u], a0 + (vi << 3), tk, ls, thr);
+      const uint32_t w[4] = {r[u].x, r[u].y, r[u].z, r[u].w};
+      float lo[4], hi[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        lo[q] = bf16_lo(w[q]);
+        hi[q] = bf16_hi(w[q]);
+        xp[u][q] = f2_pack(lo[q], hi[q]);
+      }
+      const float g = fmaxf(max3f(lo[0], hi[0], lo[1]), max3f(max3f(hi[1], lo[2], hi[2]), lo[3], hi[3]));
+      gmv[u] = (FULL || wb + lane + u * kThreads < ve) ? g : -INFINITY;
+    }
+    if constexpr (LSE) {
+      float gl = gmv[0];
+#pragma unroll
+      for (int u = 1; u < kUnroll; ++u) gl = fmaxf(gl, gmv[u]);
+      if (__any_sync(0xffffffffu, gl * kLog2e > mbw + 8.f)) {
+        const float nb = warp_max(gl) * kLog2e;
+        if (mbw != -INFINITY) {
+          const float sc = ex2(mbw - nb);
+          sacc = f2_mul(sacc, f2_pack(sc, sc));
+        }
+        mbw = nb;
+      }
+      if (mbw != -INFINITY) {
+        const uint64_t l2 = f2_pack(kLog2e, kLog2e), nb2 = f2_pack(-mbw, -mbw);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          if (FULL || wb + lane + u * kThreads < ve) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float a, b;
+              f2_unpack(f2_fma(xp[u][q], l2, nb2), a, b);
+              sacc = f2_add(sacc, f2_pack(ex2(a), ex2(b)));
+            }
+          }
+        }
+      }
+    }
+    if (wb == wb0) {
+      // first step: the k-th largest of the lanes' maxima of this step is a
+      // valid threshold already (each of those maxima is in its lane's list
+      // after the inserts below, or that lane holds k values above it), so
+      // that a warp does not start by inserting every logit it sees
+      float gl = gmv[0];
+#pragma unroll
+      for (int u = 1; u < kUnroll; ++u) gl = fmaxf(gl, gmv[u]);
+#pragma unroll
+      for (int k = 0; k < KT; ++k) {
+        const float mk = warp_max(gl);
+        if (k == KT - 1) thr = fmaxf(thr, mk);
+        if (gl == mk) gl = -INFINITY;
+      }
+    }
+    bool cand = false;
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) cand |= (FULL || wb + lane + u * kThreads < ve) && gmv[u] >= thr;
+    if (__any_sync(0xffffffffu, cand)) {
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        if ((FULL || wb + lane + u * kThreads < ve) && gmv[u] >= thr) {
+          const int idx = a0 + ((wb + lane + u * kThreads) << 3);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            float a, b;
+            f2_unpack(xp[u][q], a, b);
+            if (a >= thr) tk.insert(a, idx + 2 * q);
+            if (b >= thr) tk.insert(b, idx + 2 * q + 1);
+          }
+        }
+      }
+      thr = warp_kth(tk);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) r[u] = nx[u];
-    float th = tk.v[KT - 1];
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) th = fmaxf(th, __shfl_xor_sync(0xffffffffu, th, off));
-    thr = th;
-  }
+  };
+  int wb = wb0;
+  for (; wb + 31 + (kUnroll - 1) * kThreads < ve; wb += kUnroll * kThreads)
+    step(wb, std::integral_constant<bool, true>());
+  for (; wb < ve; wb += kUnroll * kThreads) step(wb, std::integral_constant<bool, false>());
+  float sa, sb2;
+  f2_unpack(sacc, sa, sb2);
+  const float s0 = sa, s1 = sb2;
+  if constexpr (LSE) lse_merge(ls, mbw, s0 + s1);
 
   // ---- warp merge
 #pragma unroll
@@ -331,13 +446,14 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   }
 }
 
-// One CTA per row once the rows alone give every SM two CTAs (merging a
-// split row costs more than it gains there); else split rows over a cluster
-// of up to 8 CTAs, keeping at least two vectors per thread in each.
+// One CTA per row once the rows alone give every SM six CTAs (24 warps, the
+// occupancy the scan needs to hide its load and exponential latencies); else
+// split rows over a cluster of up to 8 CTAs, keeping at least two vectors per
+// thread in each.
 int pick_split(int64_t rows, int vocab) {
   const int nvec = vocab / 8;
-  if (rows >= 2LL * num_sms()) return 1;
-  int s = (int)((4LL * num_sms() + rows - 1) / rows);
+  if (rows >= 6LL * num_sms()) return 1;
+  int s = (int)((6LL * num_sms() + rows - 1) / rows);
   s = max(1, min(s, 8));
   while (s > 1 && nvec / s < 2 * kThreads) --s;
   return s;
