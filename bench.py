@@ -222,6 +222,10 @@ def algorithmic(wl):
                 argmax_bytes=argmax_bytes, mean_nodes=float(n.mean()))
 
 
+def w_heads_kv(wl):
+    return wl["w"].heads_kv
+
+
 def resync_bytes(acc_len, layers, Hkv, D=128):
     rows = int((acc_len.astype(np.int64) + 1).sum())
     return 2 * 2 * rows * layers * Hkv * D * 2   # read + write, K and V
@@ -349,6 +353,7 @@ def main():
     Ly = wl["layers"]
     ev_attn = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * Ly)] for _ in range(args.steps)]
     ev_scan = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    ev_rs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
 
     def timed_step(s):
         e = ev_scan[s]
@@ -365,8 +370,10 @@ def main():
                                 workspace=st.workspace)
             ea[2 * l + 1].record(stream)
         acc = cure.cure_accept(tree, st.K, target_logits=x.target_logits, targ=st.targ, out=st.acc)
+        ev_rs[s][0].record(stream)
         cure.cure_resync_kv(kcs, vcs, st.kv, x.tree_k, x.tree_v, acc, x.cache_len, st.K,
                             cache_len_out=st.cache_len_out, out=st.rs)
+        ev_rs[s][1].record(stream)
 
     clk = ClockSampler(local)
     clk.start()
@@ -391,6 +398,8 @@ def main():
     assert cure.cure_device_error() == 0
     attn_ms = [ev_attn[s][2 * l].elapsed_time(ev_attn[s][2 * l + 1]) for s in range(args.steps) for l in range(Ly)]
     scan_ms = [ev_scan[s][0].elapsed_time(ev_scan[s][1]) for s in range(args.steps)]
+    rs_ms = float(np.mean([ev_rs[s][0].elapsed_time(ev_rs[s][1]) for s in range(args.steps)]))
+    rs_b = resync_bytes(acc_len, Ly, w_heads_kv(wl))
     attn_avg = float(np.mean(attn_ms))
     scan_avg = float(np.mean(scan_ms))
 
@@ -435,6 +444,9 @@ def main():
         "roofline": roof,
         "stages": {"vocab_scan_ms": round(scan_avg, 4), "vocab_scan_gbs": round(scan_gbs, 1),
                    "vocab_scan_frac": round(scan_gbs / pk["hbm_gbs"], 4),
+                   "resync_call_ms": round(rs_ms, 4),
+                   "resync_call_gbs": round(rs_b / (rs_ms * 1e-3) / 1e9, 1),
+                   "resync_call_frac": round(rs_b / (rs_ms * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
                    "tree_attn_ms_per_layer": round(attn_avg, 4),
                    "tree_attn_tflops": round(attn_tflops, 1), "tree_attn_intensity_flop_per_byte": round(intensity, 1),
                    "mean_tree_nodes": alg["mean_nodes"], "mean_accept_len": float(acc_len.mean())},

@@ -17,6 +17,7 @@ struct AttnArgs {
   const uint64_t* anc;
   int batch, n_max, heads_q, G, W, cap;
   int units_max;   // piece counters in the workspace
+  int unit_cost;   // fixed cost of a unit in the stream-K split, in 64-key tile times
   float scale_log2;
   int* cnt;        // [units_max] pieces of each unit merged so far (zero between launches)
   float* ws_o;     // [units_max + kAttnMaxCtas][32][256] float4 partial outputs
@@ -30,6 +31,13 @@ constexpr int kAttnRowsCta = 128; // query rows (node x group head) per CTA
 constexpr int kAttnKeys = 64;     // keys per tile
 constexpr int kAttnMaxBatch = 256;  // sequences per call (the CTA keeps per-sequence prefix sums)
 constexpr int kAttnMaxCtas = 256;   // persistent CTAs (one per SM, at most this many)
+// Fixed cost of a unit (its piece start-up, epilogue and split merge) in
+// 64-key tile times, charged in the stream-K split so that CTAs starting
+// more units get fewer tiles.
+#ifndef CURE_ATTN_UNIT_COST
+#define CURE_ATTN_UNIT_COST 4
+#endif
+constexpr int kAttnUnitCost = CURE_ATTN_UNIT_COST;
 
 // The persistent tcgen05 kernel (writes `out`; merges split units itself).
 cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s);

@@ -55,6 +55,7 @@ cudaError_t launch_tree_attn(const AttnPlan& plan, const uint16_t* q, const uint
   A.W = (n_max + 63) / 64;
   A.cap = kv.layout == 0 ? kv.max_len : kv.max_len * kv.page_size;
   A.units_max = plan.units_max;
+  A.unit_cost = kAttnUnitCost;
   A.scale_log2 = scale * 1.4426950408889634f;
   char* ws = reinterpret_cast<char*>(workspace);
   A.cnt = reinterpret_cast<int*>(ws);

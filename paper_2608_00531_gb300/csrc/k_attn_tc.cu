@@ -149,20 +149,28 @@ struct Seg {
   int L, n;        // cache length, tree nodes
   int part, parts; // piece index and piece count of the unit
   int slot;        // first workspace slot of the unit
+  long long next;  // cost position after the piece
 };
 
+// Work is laid out in cost positions: each unit takes C positions of fixed
+// cost (its piece start-up, epilogue and merge, in tile times) followed by
+// one position per 64-key tile.  The CTA ranges split the cost positions
+// evenly, so a CTA that starts more units gets fewer tiles.
 struct Sched {
-  const int* tiles_start;  // smem [B+1]
+  const int* tiles_start;  // smem [B+1]: first cost position of each sequence's units
   const int* units_start;  // smem [B+1]
-  int B, Hkv, P;
-  long long Ttot;
+  int B, Hkv, P, C;
+  long long Ttot;          // total cost positions
   const int* cache_len;
   const int* n_nodes;
   int cap, n_max;
-  __device__ int owner(long long g) const {  // the CTA whose range holds tile g
+  __device__ int owner(long long g) const {  // the CTA whose range holds position g
     return (int)(((g + 1) * (long long)P - 1) / Ttot);
   }
-  // The piece that starts at global tile g and ends no later than g_end.
+  // The piece that starts at cost position g (or at the first tile after it,
+  // when g is one of a unit's fixed-cost positions) and ends no later than
+  // g_end; s.next is the position after it.  s.t0 == s.t1 when the range
+  // holds no tile of that unit.
   __device__ Seg at(long long g, long long g_end) const {
     int lo = 0, hi = B;  // largest b with tiles_start[b] <= g
     while (hi - lo > 1) {
@@ -177,16 +185,20 @@ struct Sched {
     s.nct = (s.L + BN - 1) / BN;
     s.T = s.nct + (s.n + BN - 1) / BN;
     const long long local = g - tiles_start[lo];
-    const int uib = (int)(local / s.T);
+    const int Tc = s.T + C;
+    const int uib = (int)(local / Tc);
     s.rg = uib / Hkv;
     s.h = uib % Hkv;
     s.u = units_start[lo] + uib;
-    s.t0 = (int)(local % s.T);
-    s.t1 = (int)min((long long)s.T, (long long)s.t0 + (g_end - g));
-    const long long ustart = g - s.t0;
+    const int o = (int)(local % Tc);
+    const long long ustart = g - o + C;  // cost position of the unit's first tile
+    const long long gs = o < C ? ustart : g;
+    s.t0 = (int)(gs - ustart);
+    s.t1 = gs < g_end ? (int)min((long long)s.T, (long long)s.t0 + (g_end - gs)) : s.t0;
+    s.next = o < C && gs >= g_end ? g_end : gs + (s.t1 - s.t0);
     const int o0 = owner(ustart), o1 = owner(ustart + s.T - 1);
     s.parts = o1 - o0 + 1;
-    s.part = owner(g) - o0;
+    s.part = owner(gs) - o0;
     s.slot = s.u + o0;
     return s;
   }
@@ -263,7 +275,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         }
         const int rg = (n + 2 * npb - 1) / (2 * npb);
         ub = rg * Hkv;
-        tb = ub * ((L + BN - 1) / BN + (n + BN - 1) / BN);
+        tb = ub * ((L + BN - 1) / BN + (n + BN - 1) / BN + A.unit_cost);
       }
       int it = tb, iu = ub;
 #pragma unroll
@@ -298,6 +310,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
   sch.units_start = units_start;
   sch.B = B;
   sch.Hkv = Hkv;
+  sch.C = A.unit_cost;
   sch.Ttot = tiles_start[B];
   // with fewer tiles than CTAs only the first Ttot CTAs take part, so that every
   // taking part owns at least one tile and a unit's pieces are its owners
@@ -322,7 +335,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     bool ok = true;
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
-      g += s.t1 - s.t0;
+      g = s.next;
+      if (s.t1 <= s.t0) continue;
       // Q of both M tiles once the previous piece's S products are done; it
       // is requested after the piece's first K/V tile, whose ring stage frees
       // up independently, so that the ring refills across the piece boundary
@@ -419,7 +433,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     bool ok = true;
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
-      g += s.t1 - s.t0;
+      g = s.next;
+      if (s.t1 <= s.t0) continue;
       const int n = s.t1 - s.t0;
       const uint32_t gk0 = gk;
       gk += (uint32_t)n;
@@ -500,7 +515,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     bool ok = true;
     for (long long g = g_begin; g < g_end;) {
       const Seg s = sch.at(g, g_end);
-      g += s.t1 - s.t0;
+      g = s.next;
+      if (s.t1 <= s.t0) continue;
       const int n = s.t1 - s.t0;
       const uint32_t gk0 = gk;
       gk += (uint32_t)n;
