@@ -126,6 +126,12 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                : "memory");
 }
 
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ void named_sync_softmax() {  // warps 0-7
   asm volatile("bar.sync 1, 256;" ::: "memory");
 }
@@ -648,14 +654,14 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       float4* pslot = reinterpret_cast<float4*>(A.ws_o) + (int64_t)(s.slot + s.part) * (32 * 2 * BM);
       uint16_t* orow =
           A.out + (((int64_t)s.b * A.n_max + min(node, A.n_max - 1)) * A.heads_q + s.h * G + gh) * D;
-      if (act && ok) {
+      if (whole) {
+        if (act && ok) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t o[32];
-          tmem_ld32(tl + kColO + m * 128 + q * 32, o);
-          tmem_wait_ld();
-          if (vrow) {
-            if (whole) {
+          for (int q = 0; q < 4; ++q) {
+            uint32_t o[32];
+            tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+            tmem_wait_ld();
+            if (vrow) {
 #pragma unroll
               for (int i = 0; i < 32; i += 8) {
                 uint4 v;
@@ -665,83 +671,122 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
                 v.w = pack_bf16(__uint_as_float(o[i + 6]) * inv, __uint_as_float(o[i + 7]) * inv);
                 *reinterpret_cast<uint4*>(orow + q * 32 + i) = v;
               }
-            } else {
-#pragma unroll
-              for (int i = 0; i < 8; ++i)
-                pslot[(q * 8 + i) * (2 * BM) + prow] =
-                    make_float4(__uint_as_float(o[4 * i]) * inv, __uint_as_float(o[4 * i + 1]) * inv,
-                                __uint_as_float(o[4 * i + 2]) * inv, __uint_as_float(o[4 * i + 3]) * inv);
             }
           }
+          tc_fence_before();
+          mbar_arrive(bar(B_OFREE + m));
         }
-        tc_fence_before();
-        mbar_arrive(bar(B_OFREE + m));
-      }
-      if (!whole) {
-        if (vrow && ok) A.ws_lse[(int64_t)(s.slot + s.part) * (2 * BM) + prow] = m_run + log2f(l_run);
-        // the CTA that completes the unit's last piece merges the pieces
-        __threadfence();
+      } else {
+        // A piece whose unit's other pieces have all published already is the
+        // last one for sure: it neither writes its own partial nor publishes,
+        // and merges with its O read straight from TMEM.  Otherwise it writes
+        // its partial, publishes (release fence + counter), and merges if the
+        // counter says it came last.  O_m is released after the merge.
+        const float lse_own = m_run + log2f(l_run);
         named_sync_softmax();
-        if (tid == 0) {
-          int last = 0;
-          if (!*abort_flag) {
-            const int old = atomicAdd(A.cnt + s.u, 1);
-            last = old == s.parts - 1;
-            if (last) A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+        if (tid == 0) *last_flag = (!*abort_flag && ld_acquire(A.cnt + s.u) == s.parts - 1) ? 2 : 0;
+        named_sync_softmax();
+        int last = *last_flag;
+        if (last != 2) {
+          if (act && ok) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              uint32_t o[32];
+              tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+              tmem_wait_ld();
+              if (vrow) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                  pslot[(q * 8 + i) * (2 * BM) + prow] =
+                      make_float4(__uint_as_float(o[4 * i]) * inv, __uint_as_float(o[4 * i + 1]) * inv,
+                                  __uint_as_float(o[4 * i + 2]) * inv, __uint_as_float(o[4 * i + 3]) * inv);
+              }
+            }
           }
-          *last_flag = last;
-        }
-        named_sync_softmax();
-        if (*last_flag && vrow) {
+          if (vrow && ok) A.ws_lse[(int64_t)(s.slot + s.part) * (2 * BM) + prow] = lse_own;
           __threadfence();
-          // O = sum_p w_p O_p with w_p = 2^(lse_p - M) / sum_q 2^(lse_q - M).
-          // Loads are batched (two pieces x eight float4 columns per thread)
-          // so that L2 latency is paid a few times per row, not per column.
+          named_sync_softmax();
+          if (tid == 0) {
+            int l = 0;
+            if (!*abort_flag) {
+              const int old = atomicAdd(A.cnt + s.u, 1);
+              l = old == s.parts - 1;
+              if (l) A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+            }
+            *last_flag = l;
+          }
+          named_sync_softmax();
+          last = *last_flag;
+        } else if (tid == 0) {
+          A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+        }
+        if (last && act && ok) {
+          __threadfence();
+          // O = sum_p w_p O_p with w_p = 2^(lse_p - M) / sum_q 2^(lse_q - M);
+          // this piece's O_p comes from TMEM, the others' from the workspace,
+          // their loads batched (two pieces x eight float4 columns per thread)
+          const int own = s.part, no = s.parts - 1;  // other pieces: k -> k < own ? k : k + 1
           const float* lse0 = A.ws_lse + (int64_t)s.slot * (2 * BM) + prow;
-          float M = -INFINITY;
-          for (int p = 0; p < s.parts; ++p) M = fmaxf(M, __ldcg(lse0 + (int64_t)p * 2 * BM));
-          float wsum = 0.f;
-          for (int p = 0; p < s.parts; ++p) wsum += ex2(__ldcg(lse0 + (int64_t)p * 2 * BM) - M);
+          float M = lse_own;
+          if (vrow)
+            for (int k = 0; k < no; ++k) M = fmaxf(M, __ldcg(lse0 + (int64_t)(k < own ? k : k + 1) * 2 * BM));
+          float wsum = ex2(lse_own - M);
+          if (vrow)
+            for (int k = 0; k < no; ++k) wsum += ex2(__ldcg(lse0 + (int64_t)(k < own ? k : k + 1) * 2 * BM) - M);
           const float winv = 1.f / wsum;
+          const float wown = ex2(lse_own - M) * winv * inv;
           const float4* base = reinterpret_cast<const float4*>(A.ws_o) + (int64_t)s.slot * (32 * 2 * BM) + prow;
 #pragma unroll 1
-          for (int c0 = 0; c0 < 32; c0 += 8) {
-            float4 acc[8];
+          for (int q = 0; q < 4; ++q) {
+            uint32_t o[32];
+            tmem_ld32(tl + kColO + m * 128 + q * 32, o);
+            tmem_wait_ld();
+            if (vrow) {
+              float4 acc[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+              for (int i = 0; i < 8; ++i)
+                acc[i] = make_float4(__uint_as_float(o[4 * i]) * wown, __uint_as_float(o[4 * i + 1]) * wown,
+                                     __uint_as_float(o[4 * i + 2]) * wown, __uint_as_float(o[4 * i + 3]) * wown);
 #pragma unroll 1
-            for (int p0 = 0; p0 < s.parts; p0 += 2) {
-              const bool two = p0 + 1 < s.parts;
-              float4 va[8], vb[8];
-              const float4* pa = base + (int64_t)p0 * (32 * 2 * BM) + c0 * (2 * BM);
+              for (int k0 = 0; k0 < no; k0 += 2) {
+                const bool two = k0 + 1 < no;
+                const int pa_i = k0 < own ? k0 : k0 + 1, pb_i = k0 + 1 < own ? k0 + 1 : k0 + 2;
+                float4 va[8], vb[8];
+                const float4* pa = base + (int64_t)pa_i * (32 * 2 * BM) + q * 8 * (2 * BM);
+                const float4* pbp = base + (int64_t)pb_i * (32 * 2 * BM) + q * 8 * (2 * BM);
 #pragma unroll
-              for (int i = 0; i < 8; ++i) va[i] = __ldcg(pa + i * (2 * BM));
-              if (two) {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) vb[i] = __ldcg(pa + 32 * 2 * BM + i * (2 * BM));
-              }
-              const float wa = ex2(__ldcg(lse0 + (int64_t)p0 * 2 * BM) - M) * winv;
-              const float wb = two ? ex2(__ldcg(lse0 + (int64_t)(p0 + 1) * 2 * BM) - M) * winv : 0.f;
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                acc[i].x += wa * va[i].x; acc[i].y += wa * va[i].y;
-                acc[i].z += wa * va[i].z; acc[i].w += wa * va[i].w;
+                for (int i = 0; i < 8; ++i) va[i] = __ldcg(pa + i * (2 * BM));
                 if (two) {
-                  acc[i].x += wb * vb[i].x; acc[i].y += wb * vb[i].y;
-                  acc[i].z += wb * vb[i].z; acc[i].w += wb * vb[i].w;
+#pragma unroll
+                  for (int i = 0; i < 8; ++i) vb[i] = __ldcg(pbp + i * (2 * BM));
+                }
+                const float wa = ex2(__ldcg(lse0 + (int64_t)pa_i * 2 * BM) - M) * winv;
+                const float wb = two ? ex2(__ldcg(lse0 + (int64_t)pb_i * 2 * BM) - M) * winv : 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                  acc[i].x += wa * va[i].x; acc[i].y += wa * va[i].y;
+                  acc[i].z += wa * va[i].z; acc[i].w += wa * va[i].w;
+                  if (two) {
+                    acc[i].x += wb * vb[i].x; acc[i].y += wb * vb[i].y;
+                    acc[i].z += wb * vb[i].z; acc[i].w += wb * vb[i].w;
+                  }
                 }
               }
-            }
 #pragma unroll
-            for (int i = 0; i < 8; i += 2) {
-              uint4 v;
-              v.x = pack_bf16(acc[i].x, acc[i].y);
-              v.y = pack_bf16(acc[i].z, acc[i].w);
-              v.z = pack_bf16(acc[i + 1].x, acc[i + 1].y);
-              v.w = pack_bf16(acc[i + 1].z, acc[i + 1].w);
-              *reinterpret_cast<uint4*>(orow + (c0 + i) * 4) = v;
+              for (int i = 0; i < 8; i += 2) {
+                uint4 v;
+                v.x = pack_bf16(acc[i].x, acc[i].y);
+                v.y = pack_bf16(acc[i].z, acc[i].w);
+                v.z = pack_bf16(acc[i + 1].x, acc[i + 1].y);
+                v.w = pack_bf16(acc[i + 1].z, acc[i + 1].w);
+                *reinterpret_cast<uint4*>(orow + q * 32 + i * 4) = v;
+              }
             }
           }
+        }
+        if (act && ok) {
+          tc_fence_before();
+          mbar_arrive(bar(B_OFREE + m));
         }
       }
     }
