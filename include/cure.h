@@ -144,7 +144,11 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
  * models; otherwise CURE_ERR_INVALID_ARG), all tensor base pointers 16-byte
  * aligned.
  * workspace: device scratch of at least cure_tree_attn_workspace_size() bytes,
- * 256-byte aligned (split-KV partial results).
+ * 256-byte aligned (split-KV partial results); its contents on entry do not
+ * matter.  Calls that can overlap on the GPU must not share a workspace.
+ * The kernel is launched as a programmatic dependent launch: it starts its
+ * set-up while the previous kernel on the stream finishes and waits for that
+ * kernel before reading any argument, so stream order is kept.
  */
 cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v,
                            const void* k_cache, const void* v_cache, const cure_kv_desc* kv,

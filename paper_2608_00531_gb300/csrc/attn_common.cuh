@@ -19,7 +19,8 @@ struct AttnArgs {
   int units_max;   // piece counters in the workspace
   int unit_cost;   // fixed cost of a unit in the stream-K split, in 64-key tile times
   float scale_log2;
-  int* cnt;        // [units_max] pieces of each unit merged so far (zero between launches)
+  int* cnt;        // [units_max] (launch tag << 9) | pieces arrived, per unit
+  uint32_t tag;    // this launch's tag (set by the launcher)
   float* ws_o;     // [units_max + kAttnMaxCtas][32][256] float4 partial outputs
   float* ws_lse;   // [(units_max + kAttnMaxCtas) * 256] partial base-2 log-sum-exps
   uint16_t* out;
@@ -35,7 +36,7 @@ constexpr int kAttnMaxCtas = 256;   // persistent CTAs (one per SM, at most this
 // 64-key tile times, charged in the stream-K split so that CTAs starting
 // more units get fewer tiles.
 #ifndef CURE_ATTN_UNIT_COST
-#define CURE_ATTN_UNIT_COST 4
+#define CURE_ATTN_UNIT_COST 3
 #endif
 constexpr int kAttnUnitCost = CURE_ATTN_UNIT_COST;
 

@@ -2,7 +2,8 @@
 // tcgen05 tree-attention kernel (k_attn_tc.cu).
 //
 // Workspace layout (caller-owned, 256-byte aligned):
-//   cnt     int32 [units_max], 256-byte rounded   pieces merged per unit
+//   cnt     int32 [units_max], 256-byte rounded   (launch tag << 9) | pieces arrived,
+//                                                 per unit (any initial contents)
 //   ws_o    fp32  [units_max + kAttnMaxCtas][32][256] float4: per piece slot, column-major
 //                 partial outputs (float4 column c of row r at [slot][c][r])
 //   ws_lse  fp32  [(units_max + kAttnMaxCtas) * 256]        partial log-sum-exps

@@ -126,6 +126,28 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                : "memory");
 }
 
+// A unit's piece counter holds (launch tag << 9) | pieces arrived.  A word
+// whose tag is not this launch's (left by an aborted launch, or never
+// written) counts as zero, so the workspace needs no reset; a completed unit
+// leaves zero behind, so an old word can only match a later tag if its launch
+// was aborted exactly 2^23 - 1 launches earlier.
+constexpr int kCountBits = 9;
+constexpr int kCountMask = (1 << kCountBits) - 1;
+__device__ __forceinline__ int count_of(int v, uint32_t tag) {
+  return ((uint32_t)v >> kCountBits) == tag ? (v & kCountMask) : 0;
+}
+// This piece's arrival (after its release fence): the pieces arrived so far,
+// this one included.
+__device__ __forceinline__ int arrive(int* cnt, uint32_t tag) {
+  int old = *reinterpret_cast<volatile int*>(cnt);
+  while (true) {
+    const int nw = (int)((tag << kCountBits) | (uint32_t)(count_of(old, tag) + 1));
+    const int prev = atomicCAS(cnt, old, nw);
+    if (prev == old) return nw & kCountMask;
+    old = prev;
+  }
+}
+
 __device__ __forceinline__ int ld_acquire(const int* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -263,6 +285,11 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     const int q16 = c & 7, rr = npb * G + ((c >> 3) % pad_rows), mh = (c >> 3) / pad_rows;
     st_shared_v4(sb + kOffQ + mh * kQHalf + rr * 128 + q16 * 16, 0u, 0u, 0u, 0u);
   }
+  // the inputs may be written by the previous kernel on the stream: wait for
+  // it (a programmatic launch lets this grid start its set-up early) before
+  // the first read, and let the next kernel start its set-up
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   // per-sequence tiles and units, and their prefix sums (warp 9 scans)
   if (warp == 9) {
     int run_t = 0, run_u = 0;
@@ -684,7 +711,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         // counter says it came last.  O_m is released after the merge.
         const float lse_own = m_run + log2f(l_run);
         named_sync_softmax();
-        if (tid == 0) *last_flag = (!*abort_flag && ld_acquire(A.cnt + s.u) == s.parts - 1) ? 2 : 0;
+        if (tid == 0)
+          *last_flag = (!*abort_flag && count_of(ld_acquire(A.cnt + s.u), A.tag) == s.parts - 1) ? 2 : 0;
         named_sync_softmax();
         int last = *last_flag;
         if (last != 2) {
@@ -709,16 +737,15 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           if (tid == 0) {
             int l = 0;
             if (!*abort_flag) {
-              const int old = atomicAdd(A.cnt + s.u, 1);
-              l = old == s.parts - 1;
-              if (l) A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+              l = arrive(A.cnt + s.u, A.tag) == s.parts;
+              if (l) A.cnt[s.u] = 0;  // a completed unit leaves a zero word behind
             }
             *last_flag = l;
           }
           named_sync_softmax();
           last = *last_flag;
         } else if (tid == 0) {
-          A.cnt[s.u] = 0;  // leave the counter ready for the next launch
+          A.cnt[s.u] = 0;  // a completed unit leaves a zero word behind
         }
         if (last && act && ok) {
           __threadfence();
@@ -870,10 +897,25 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
   ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_kv_map(&mtv, A.tv, trows, Hkv, BN) &&
        make_q_map(&mq, A.q, trows, Hkv, A.G, BM / A.G);
   if (!ok) return cudaErrorInvalidValue;
-  // the per-unit piece counters start at zero (the kernel leaves them at zero)
-  e = cudaMemsetAsync(A.cnt, 0, sizeof(int) * (size_t)A.units_max, s);
+  // a fresh tag per launch makes the piece counters left in the workspace
+  // count as zero (1 .. 2^23 - 1; zero-filled memory is never current)
+  static std::atomic<uint32_t> launches{0};
+  AttnArgs a = A;
+  a.tag = launches.fetch_add(1) % ((1u << (32 - kCountBits)) - 1) + 1;
+  // a programmatic launch: the kernel waits for the previous grid before it
+  // reads anything, so only its set-up overlaps that grid's tail
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel, mk, mv, mtk, mtv, mq, a);
   if (e != cudaSuccess) return e;
-  tree_attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(mk, mv, mtk, mtv, mq, A);
   return cudaGetLastError();
 }
 
