@@ -465,25 +465,25 @@ def main():
 
 
 def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
-    """Same step through the public API with inputs in pinned host memory:
-    host-to-device copies of the step's inputs and a device-to-host read of
-    the accept results inside the timed region.  Whole-job value over ranks."""
+    """Same step through the public API with inputs in pinned host memory
+    (RepairVerifyStep.run_from_host): host-to-device copies of the step's
+    inputs and a device-to-host read of the accept results inside the timed
+    region.  Whole-job value over ranks."""
     from paper_2608_00531_gb300.step import StepInputs
     x = wl["x"]
     host = {k_: getattr(x, k_).cpu().pin_memory() for k_ in ("draft_logits", "root_tok", "cache_len", "q",
                                                                "tree_k", "tree_v", "target_logits")}
-    dbuf = {k_: torch.empty_like(v, device=dev) for k_, v in host.items()}
     outs = torch.empty(4, st.B, st.K + 2, dtype=torch.int32).pin_memory()
     h2d = sum(v.numel() * v.element_size() for v in host.values())
     d2h = outs.numel() * outs.element_size()
     stream = torch.cuda.current_stream()
+    xh = StepInputs(host["draft_logits"], host["root_tok"], host["cache_len"], None, host["q"], host["tree_k"],
+                    host["tree_v"], host["target_logits"])
 
     def one():
-        for k_, v in host.items():
-            dbuf[k_].copy_(v, non_blocking=True)
-        xi = StepInputs(dbuf["draft_logits"], dbuf["root_tok"], dbuf["cache_len"], None, dbuf["q"],
-                        dbuf["tree_k"], dbuf["tree_v"], dbuf["target_logits"])
-        r = st.run(xi, kcs, vcs)
+        # the public step with host inputs: it streams them in on a copy
+        # stream, each stage waiting for its own inputs
+        r = st.run_from_host(xh, kcs, vcs)
         outs[0, :, 0].copy_(r["acc"]["accept_len"], non_blocking=True)
         outs[1].copy_(r["acc"]["out_tokens"], non_blocking=True)
         outs[2].copy_(r["resync"]["replay_tokens"], non_blocking=True)

@@ -9,6 +9,11 @@ on one stream:
 Inputs of a step (``StepInputs``) are the draft logits, the tree's target
 Q/K/V per layer and the target logits; the KV caches are persistent state
 owned by the caller.  Nothing here computes: every stage is a libcure call.
+
+``run_from_host`` takes the same inputs in (pinned) host memory and streams
+them in on a copy stream in the order the stages consume them (draft logits,
+then each layer's Q/K/V, then the target logits); each stage waits only for
+its own inputs, so the copies overlap the stages before them.
 """
 from __future__ import annotations
 
@@ -69,6 +74,8 @@ class RepairVerifyStep:
         self.rs = dict(draft_valid_len=torch.empty(B, **i32), replay_tokens=torch.empty(B, P, **i32),
                        n_replay=torch.empty(B, **i32))
         self.cache_len_out = torch.empty(B, **i32)
+        self._dev_inputs = None
+        self._copy_stream = None
 
     def run(self, x: StepInputs, k_caches: List[torch.Tensor], v_caches: List[torch.Tensor],
             stream=None) -> dict:
@@ -88,6 +95,59 @@ class RepairVerifyStep:
         vl = [v_caches[self.layer_map[l]] for l in range(self.layers)]
         rs = cure.cure_resync_kv(kl, vl, self.kv, x.tree_k, x.tree_v, acc, x.cache_len, self.K,
                                  cache_len_out=self.cache_len_out, out=self.rs, stream=stream)
+        return dict(score=self.score, tree=tree, attn=self.attn_out, acc=acc, resync=rs)
+
+    def run_from_host(self, xh: StepInputs, k_caches: List[torch.Tensor], v_caches: List[torch.Tensor],
+                      stream=None) -> dict:
+        """One step with its inputs in host memory (pinned, for copies that
+        overlap the stages): copies on a side stream, each stage waiting for
+        the copy of its own inputs.  Results stay on the device, as in run()."""
+        fields = ("draft_logits", "root_tok", "cache_len", "q", "tree_k", "tree_v", "target_logits")
+        dev = self.attn_out.device
+        if self._dev_inputs is None or any(self._dev_inputs[f].shape != getattr(xh, f).shape for f in fields):
+            self._dev_inputs = {f: torch.empty(getattr(xh, f).shape, dtype=getattr(xh, f).dtype, device=dev)
+                                for f in fields}
+            self._copy_stream = torch.cuda.Stream(device=dev)
+        d = self._dev_inputs
+        main = stream if stream is not None else torch.cuda.current_stream(dev)
+        cs = self._copy_stream
+        cs.wait_stream(main)  # the previous step's reads of the staging buffers come first
+        ev_first = torch.cuda.Event()
+        ev_layer = [torch.cuda.Event() for _ in range(self.layers)]
+        ev_target = torch.cuda.Event()
+        with torch.cuda.stream(cs):
+            for f in ("draft_logits", "root_tok", "cache_len"):
+                d[f].copy_(getattr(xh, f), non_blocking=True)
+            ev_first.record(cs)
+            for l in range(self.layers):
+                for f in ("q", "tree_k", "tree_v"):
+                    d[f][l].copy_(getattr(xh, f)[l], non_blocking=True)
+                ev_layer[l].record(cs)
+            d["target_logits"].copy_(xh.target_logits, non_blocking=True)
+            ev_target.record(cs)
+        x = StepInputs(d["draft_logits"], d["root_tok"], d["cache_len"], None if xh.redraft is None else
+                       xh.redraft.to(dev, non_blocking=True), d["q"], d["tree_k"], d["tree_v"],
+                       d["target_logits"])
+        with torch.cuda.stream(main):
+            main.wait_event(ev_first)
+            ids, vals, margin, logp1 = cure.cure_score_draft(x.draft_logits, self.k, out=self.score,
+                                                             stream=main)
+            tree = cure.cure_build_tree(ids, margin, x.root_tok, x.cache_len, self.tau, self.R,
+                                        self.branches, self.depth, x.redraft, self.max_ufp,
+                                        out=self.tree, stream=main)
+            for l in range(self.layers):
+                main.wait_event(ev_layer[l])
+                p = self.layer_map[l]
+                cure.cure_tree_attn(x.q[l], x.tree_k[l], x.tree_v[l], k_caches[p], v_caches[p], self.kv,
+                                    x.cache_len, tree["n_nodes"], tree["anc"], self.scale,
+                                    out=self.attn_out[l], workspace=self.workspace, stream=main)
+            main.wait_event(ev_target)
+            acc = cure.cure_accept(tree, self.K, target_logits=x.target_logits, targ=self.targ,
+                                   out=self.acc, stream=main)
+            kl = [k_caches[self.layer_map[l]] for l in range(self.layers)]
+            vl = [v_caches[self.layer_map[l]] for l in range(self.layers)]
+            rs = cure.cure_resync_kv(kl, vl, self.kv, x.tree_k, x.tree_v, acc, x.cache_len, self.K,
+                                     cache_len_out=self.cache_len_out, out=self.rs, stream=main)
         return dict(score=self.score, tree=tree, attn=self.attn_out, acc=acc, resync=rs)
 
     @property

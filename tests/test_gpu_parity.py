@@ -490,3 +490,22 @@ def test_full_step_serve_shape(cure):
     for l in range(layers):
         assert np.array_equal(_f64(kcs[l].cpu()), kc_host[l])
         assert np.array_equal(_f64(vcs[l].cpu()), vc_host[l])
+    # the same step with its inputs in pinned host memory, streamed in on a
+    # copy stream: the same results (the step's buffers are reused, so the
+    # first results are copied out first)
+    ints = {("tree", k_): v.clone() for k_, v in r["tree"].items()}
+    ints.update({("acc", k_): v.clone() for k_, v in r["acc"].items()})
+    ints.update({("resync", k_): v.clone() for k_, v in r["resync"].items()})
+    attn = r["attn"].float().clone()
+    xh = StepInputs(d.logits.pin_memory(), torch.from_numpy(d.root_tok).pin_memory(),
+                    torch.from_numpy(L).pin_memory(), None, q.pin_memory(), tk.pin_memory(), tv.pin_memory(),
+                    tl.pin_memory())
+    for _ in range(2):
+        r2 = st.run_from_host(xh, kcs, vcs)
+        torch.cuda.synchronize()
+        assert cure.cure_device_error() == 0
+        for (grp, key), v in ints.items():
+            assert torch.equal(r2[grp][key], v), (grp, key)
+        for b in range(B):
+            nb = int(t["n_nodes"][b])
+            assert float((r2["attn"][:, b, :nb].float() - attn[:, b, :nb]).abs().max()) <= 1e-2, b
