@@ -20,6 +20,33 @@ __device__ __forceinline__ void flag(int* err, int bits) {
   if (err) atomicOr(err, bits);
 }
 
+// ---- programmatic dependent launch ----
+// The library's kernels are launched so that each may be scheduled while the
+// previous kernel on the stream finishes (its set-up then overlaps that
+// kernel's tail); every kernel calls pdl_begin() before its first read of
+// global memory, which waits for the previous kernel to complete and lets
+// the next one be scheduled.  Without a programmatic launch both are no-ops.
+__device__ __forceinline__ void pdl_begin() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // ---- launchers (all asynchronous on `s`; return the launch's cudaError_t) ----
 cudaError_t launch_score(const uint16_t* logits, int64_t rows, int vocab, int topk,
                          int32_t* top_ids, float* top_vals, float* margin, float* logp1,

@@ -285,11 +285,9 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     const int q16 = c & 7, rr = npb * G + ((c >> 3) % pad_rows), mh = (c >> 3) / pad_rows;
     st_shared_v4(sb + kOffQ + mh * kQHalf + rr * 128 + q16 * 16, 0u, 0u, 0u, 0u);
   }
-  // the inputs may be written by the previous kernel on the stream: wait for
-  // it (a programmatic launch lets this grid start its set-up early) before
-  // the first read, and let the next kernel start its set-up
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // the set-up above reads no global memory; wait for the previous kernel on
+  // the stream before the first read (programmatic dependent launch)
+  pdl_begin();
   // per-sequence tiles and units, and their prefix sums (warp 9 scans)
   if (warp == 9) {
     int run_t = 0, run_u = 0;
@@ -902,19 +900,7 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
   static std::atomic<uint32_t> launches{0};
   AttnArgs a = A;
   a.tag = launches.fetch_add(1) % ((1u << (32 - kCountBits)) - 1) + 1;
-  // a programmatic launch: the kernel waits for the previous grid before it
-  // reads anything, so only its set-up overlaps that grid's tail
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel, mk, mv, mtk, mtv, mq, a);
+  e = launch_pdl(tree_attn_tc_kernel, grid, dim3(kThreads), kSmemBytes, s, mk, mv, mtk, mtv, mq, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -17,6 +17,7 @@ resync_gather_kernel(int layers, LayerPtrs caches, cure_kv_desc kv, const uint4*
                      const uint4* __restrict__ tree_v, int batch, int n_max, int block,
                      const int32_t* __restrict__ path_nodes, const int32_t* __restrict__ accept_len,
                      const int32_t* __restrict__ cache_len_in, int* err) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const int T = block + 1;                      // depths 0..K
   const int64_t item = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
@@ -70,6 +71,7 @@ __global__ void resync_finalize_kernel(int batch, int block, const int32_t* __re
                                        int32_t* __restrict__ draft_valid_len,
                                        int32_t* __restrict__ replay_tokens,
                                        int32_t* __restrict__ n_replay) {
+  pdl_begin();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
   const int P = block + 2;
@@ -103,16 +105,15 @@ cudaError_t launch_resync(int layers, const LayerPtrs& caches, const cure_kv_des
   if (layers > 0) {
     const int64_t items = (int64_t)layers * 2 * batch * (block + 1);
     const int64_t grid = (items + kWarps - 1) / kWarps;
-    resync_gather_kernel<<<(unsigned)grid, 32 * kWarps, 0, s>>>(
-        layers, caches, kv, reinterpret_cast<const uint4*>(tree_k), reinterpret_cast<const uint4*>(tree_v),
-        batch, n_max, block, path_nodes, accept_len, cache_len_in, err);
-    const cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_pdl(
+        resync_gather_kernel, dim3((unsigned)grid), dim3(32 * kWarps), 0, s, layers, caches, kv,
+        reinterpret_cast<const uint4*>(tree_k), reinterpret_cast<const uint4*>(tree_v), batch, n_max,
+        block, path_nodes, accept_len, cache_len_in, err);
     if (e != cudaSuccess) return e;
   }
-  resync_finalize_kernel<<<(batch + 127) / 128, 128, 0, s>>>(batch, block, accept_len, diverge_depth,
-                                                            out_tokens, cache_len_in, cache_len_out,
-                                                            draft_valid_len, replay_tokens, n_replay);
-  return cudaGetLastError();
+  return launch_pdl(resync_finalize_kernel, dim3((batch + 127) / 128), dim3(128), 0, s, batch, block,
+                    accept_len, diverge_depth, out_tokens, cache_len_in, cache_len_out, draft_valid_len,
+                    replay_tokens, n_replay);
 }
 
 }  // namespace cure

@@ -42,6 +42,7 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
                   int32_t* __restrict__ parent, int32_t* __restrict__ depth,
                   uint64_t* __restrict__ anc, int32_t* __restrict__ ufp_pos,
                   int32_t* __restrict__ n_ufp) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
   const int b = blockIdx.x * kWarpsPerCta + wib;
@@ -172,6 +173,7 @@ accept_walk_kernel(int batch, int n_max, int block, const int32_t* __restrict__ 
                    int32_t* __restrict__ best_node, int32_t* __restrict__ path_nodes,
                    int32_t* __restrict__ out_tokens, int32_t* __restrict__ diverge_depth,
                    int* err) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
   const int b = blockIdx.x * kWarpsPerCta + wib;
@@ -262,10 +264,9 @@ cudaError_t launch_build_tree(const cure_tree_params& p, const int32_t* top_ids,
   (void)err;
   if (p.batch == 0) return cudaSuccess;
   const int grid = (p.batch + kWarpsPerCta - 1) / kWarpsPerCta;
-  build_tree_kernel<<<grid, 32 * kWarpsPerCta, 0, s>>>(p, top_ids, margin, root_tok, cache_len,
-                                                       redraft, n_nodes, tok, pos, parent, depth,
-                                                       anc, ufp_pos, n_ufp);
-  return cudaGetLastError();
+  return launch_pdl(build_tree_kernel, dim3(grid), dim3(32 * kWarpsPerCta), 0, s, p, top_ids, margin,
+                    root_tok, cache_len, redraft, n_nodes, tok, pos, parent, depth, anc, ufp_pos,
+                    n_ufp);
 }
 
 cudaError_t launch_accept_walk(int batch, int n_max, int block, const int32_t* n_nodes,
@@ -275,11 +276,9 @@ cudaError_t launch_accept_walk(int batch, int n_max, int block, const int32_t* n
                                int32_t* diverge_depth, int* err, cudaStream_t s) {
   if (batch == 0) return cudaSuccess;
   const int grid = (batch + kWarpsPerCta - 1) / kWarpsPerCta;
-  accept_walk_kernel<<<grid, 32 * kWarpsPerCta, 0, s>>>(batch, n_max, block, n_nodes, tok,
-                                                        parent, depth, anc, targ, accept_len,
-                                                        best_node, path_nodes, out_tokens,
-                                                        diverge_depth, err);
-  return cudaGetLastError();
+  return launch_pdl(accept_walk_kernel, dim3(grid), dim3(32 * kWarpsPerCta), 0, s, batch, n_max, block,
+                    n_nodes, tok, parent, depth, anc, targ, accept_len, best_node, path_nodes,
+                    out_tokens, diverge_depth, err);
 }
 
 }  // namespace cure

@@ -198,6 +198,7 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
                   const int32_t* __restrict__ n_nodes, int32_t* __restrict__ top_ids,
                   float* __restrict__ top_vals, float* __restrict__ margin,
                   float* __restrict__ logp1) {
+  pdl_begin();
   const int64_t row = blockIdx.y;
   const int S = gridDim.x;
   const int c = blockIdx.x;  // rank within the cluster
@@ -469,13 +470,15 @@ cudaError_t launch_scan(const uint16_t* logits, int64_t rows, int vocab, int k_o
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see pdl_begin()
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, vocab_scan_kernel<KT, LSE, TARGET>, logits, vocab, k_out,
                             n_max, n_nodes, top_ids, top_vals, margin, logp1);
 }
