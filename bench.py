@@ -166,14 +166,16 @@ def job_steps_per_s(ms_max: float, steps: int, world: int) -> float:
 
 
 # ------------------------------------------------------------------ workload
-def make_workload(dev, rank: int, layers_override=None):
+POOL = 4  # draft/target input sets cycled over the steps, so that tree shapes vary
+
+
+def make_workload(dev, rank: int, layers_override=None, pool: int = POOL):
     from paper_2608_00531_gb300 import cure, workload as W
     from paper_2608_00531_gb300.step import RepairVerifyStep, StepInputs
     w = W.WORKLOADS[WORKLOAD]
     seed = rank_seed(w.seed, rank)
     layers = layers_override or w.layers
     B, K, N, D = w.batch, w.block, w.n_max, 128
-    d = W.draft_block(w, seed=seed)
     L = W.cache_lengths(w, seed=seed)
     table, npages = W.block_table(L, K, seed)
     g = torch.Generator(device=dev).manual_seed(seed)
@@ -189,25 +191,33 @@ def make_workload(dev, rank: int, layers_override=None):
     bt = torch.from_numpy(table).to(dev)
     kv = cure.kv_desc(w.heads_kv, D, table.shape[1], bt, 16, npages)
     st = RepairVerifyStep(B, K, w.vocab, w.topk, w.tau, w.budget, w.branches, 1, layers, w.heads_q, kv, dev)
-    draft = d.logits.to(dev)
-    root = torch.from_numpy(d.root_tok).to(dev)
     lens = torch.from_numpy(L).to(dev)
-    # the target's logits come from a stand-in target model applied to the
-    # tree this batch produces (built once, outside the timed region)
-    ids, vals, margin, lp = cure.cure_score_draft(draft, w.topk)
-    tree = cure.cure_build_tree(ids, margin, root, lens, w.tau, w.budget, w.branches)
-    th = {k_: v.cpu().numpy() for k_, v in tree.items()}
-    truth = W.target_truth(w, d, seed)
-    targ = W.synthetic_target_ids(truth, th["n_nodes"], th["tok"], th["parent"], th["depth"], w.vocab, seed)
-    tl = W.target_logits(targ, w.vocab, seed).to(dev)
-    x = StepInputs(draft, root, lens, None, q, tk, tv, tl)
-    return dict(w=w, st=st, x=x, kcs=kcs, vcs=vcs, kv=kv, L=L, tree=th, d=d, seed=seed, layers=layers,
-                npages=npages, table=table)
+    xs, trees = [], []
+    for i in range(pool):
+        # each set: its own draft block (so its own tree) and target; the
+        # target's logits come from a stand-in target model applied to the
+        # tree the set produces (built once here, outside the timed region)
+        si = seed + 1009 * i
+        d = W.draft_block(w, seed=si)
+        draft = d.logits.to(dev)
+        root = torch.from_numpy(d.root_tok).to(dev)
+        ids, vals, margin, lp = cure.cure_score_draft(draft, w.topk)
+        tree = cure.cure_build_tree(ids, margin, root, lens, w.tau, w.budget, w.branches)
+        th = {k_: v.cpu().numpy() for k_, v in tree.items()}
+        truth = W.target_truth(w, d, si)
+        targ = W.synthetic_target_ids(truth, th["n_nodes"], th["tok"], th["parent"], th["depth"], w.vocab, si)
+        tl = W.target_logits(targ, w.vocab, si).to(dev)
+        xs.append(StepInputs(draft, root, lens, None, q, tk, tv, tl))
+        trees.append(th)
+    return dict(w=w, st=st, x=xs[0], xs=xs, kcs=kcs, vcs=vcs, kv=kv, L=L, tree=trees[0], trees=trees, seed=seed,
+                layers=layers, npages=npages, table=table)
 
 
-def algorithmic(wl):
-    """Bytes and flops the method must move or compute per step, per stage."""
-    w, th, L = wl["w"], wl["tree"], wl["L"].astype(np.int64)
+def algorithmic(wl, th=None):
+    """Bytes and flops the method must move or compute per step, per stage
+    (for the input set whose tree is th)."""
+    w, L = wl["w"], wl["L"].astype(np.int64)
+    th = wl["tree"] if th is None else th
     B, K, N, V, D = w.batch, w.block, w.n_max, w.vocab, 128
     Hq, Hkv, layers = w.heads_q, w.heads_kv, wl["layers"]
     n = th["n_nodes"].astype(np.int64)
@@ -314,6 +324,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help=argparse.SUPPRESS)
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
@@ -339,15 +350,20 @@ def main():
     from paper_2608_00531_gb300 import cure
 
     wl = make_workload(dev, rank, args.layers)
-    st, x, kcs, vcs = wl["st"], wl["x"], wl["kcs"], wl["vcs"]
+    st, xs, kcs, vcs = wl["st"], wl["xs"], wl["kcs"], wl["vcs"]
+    P = len(xs)
     stream = torch.cuda.current_stream()
 
-    for _ in range(args.warmup):
-        r = st.run(x, kcs, vcs)
-    torch.cuda.synchronize()
+    acc_lens = [None] * P
+    for i in range(max(args.warmup, P)):
+        r = st.run(xs[i % P], kcs, vcs)
+        torch.cuda.synchronize()
+        acc_lens[i % P] = r["acc"]["accept_len"].cpu().numpy()
     assert cure.cure_device_error() == 0
-    acc_len = r["acc"]["accept_len"].cpu().numpy()
-    alg = algorithmic(wl)
+    algs = [algorithmic(wl, th) for th in wl["trees"]]
+    # the timed steps cycle over the sets: per-step averages
+    sel = [s % P for s in range(args.steps)]
+    alg = {k_: float(np.mean([algs[i][k_] for i in sel])) for k_ in algs[0]}
 
     # per-op events inside the timed region (same stream as the launches)
     Ly = wl["layers"]
@@ -359,6 +375,7 @@ def main():
     ev_rs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
 
     def timed_step(s):
+        x = xs[s % P]
         e = ev_scan[s]
         e[0].record(stream)
         cure.cure_score_draft(x.draft_logits, st.k, out=st.score)
@@ -402,9 +419,14 @@ def main():
     attn_ms = [ev_attn[s][0].elapsed_time(ev_attn[s][1]) / Ly for s in range(args.steps)]
     scan_ms = [ev_scan[s][0].elapsed_time(ev_scan[s][1]) for s in range(args.steps)]
     rs_ms = float(np.mean([ev_rs[s][0].elapsed_time(ev_rs[s][1]) for s in range(args.steps)]))
-    rs_b = resync_bytes(acc_len, Ly, w_heads_kv(wl))
+    rs_b = float(np.mean([resync_bytes(acc_lens[i], Ly, w_heads_kv(wl)) for i in sel]))
     attn_avg = float(np.mean(attn_ms))
     scan_avg = float(np.mean(scan_ms))
+
+    # the same step replayed as CUDA graphs (one per input set), timed the same way
+    graph = None
+    if not args.no_graph:
+        graph = run_graphs(st, xs, kcs, vcs, args.steps, world, dev)
 
     # end to end through the public API with host buffers
     e2e = None
@@ -453,15 +475,57 @@ def main():
                    "resync_call_frac": round(rs_b / (rs_ms * 1e-3) / 1e9 / pk["hbm_gbs"], 4),
                    "tree_attn_ms_per_layer": round(attn_avg, 4),
                    "tree_attn_tflops": round(attn_tflops, 1), "tree_attn_intensity_flop_per_byte": round(intensity, 1),
-                   "mean_tree_nodes": alg["mean_nodes"], "mean_accept_len": float(acc_len.mean())},
+                   "mean_tree_nodes": round(alg["mean_nodes"], 3),
+                   "mean_accept_len": round(float(np.mean([acc_lens[i].mean() for i in sel])), 3),
+                   "input_sets": P},
         "gpu_launches": st.launches_per_step * args.steps,
         "clocks": clocks,
     }
     if e2e:
         out["e2e"] = e2e
+    if graph:
+        out["graph"] = graph
     if not args.no_cpu_baseline and world == 1:
         out["cpu_baseline"] = cpu_baseline()
     print(json.dumps(out), flush=True)
+
+
+def run_graphs(st, xs, kcs, vcs, steps, world, dev):
+    """The step captured once per input set as a CUDA graph (launches and
+    their programmatic edges recorded) and replayed, cycling over the sets."""
+    try:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            for x in xs:
+                st.run(x, kcs, vcs)
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        graphs = []
+        for x in xs:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                st.run(x, kcs, vcs)
+            graphs.append(g)
+        for g in graphs:
+            g.replay()
+        torch.cuda.synchronize()
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        stream = torch.cuda.current_stream()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for s in range(steps):
+            graphs[s % len(graphs)].replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = max_over_ranks(a.elapsed_time(b), world, dev) / steps
+        return {"value": round(job_steps_per_s(ms * steps, steps, world), 3), "unit": "steps/s",
+                "ms_per_step": round(ms, 4), "steps": steps}
+    except Exception as e:  # report, do not fail the bench line
+        return {"error": f"{type(e).__name__}: {e}"[:200]}
 
 
 def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
