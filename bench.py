@@ -35,7 +35,7 @@ import torch  # noqa: E402
 # DRAM bytes (read + write) of one tree-attention launch on this workload, from
 # one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
 # source with the given sha256 prefix; another source reports null
-ATTN_TRAFFIC = {"c0c086d83a995ea5": 313_532_416}
+ATTN_TRAFFIC = {"f7b619d89bf865b0": 313165312}
 
 METRIC = "repair-verify steps/s at batch 32, block 16; tree-attn & vocab-scan HBM GB/s vs peak"
 WORKLOAD = "serve32"
