@@ -107,6 +107,27 @@ __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatil
   return __all_sync(0xffffffffu, ok);
 }
 
+// Pairs of floats in one 64-bit register pair, for the packed f32x2
+// arithmetic of sm_100 and later (two lanes of work per instruction).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // max of three (sm_100 and later have a three-input float max)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
@@ -611,14 +632,21 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           const bool need = m_new > m_run + 8.0f;
           const float m_use = need ? m_new : m_run;
           const float nbase = m_use == -INFINITY ? 0.f : -m_use;
+          // exponent arguments and row sums two at a time (packed f32x2)
           uint32_t pk[32];
-          float sm[4] = {0.f, 0.f, 0.f, 0.f};
+          const uint64_t c2 = f2_pack(c, c), nb2 = f2_pack(nbase, nbase);
+          uint64_t sm2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float p0 = ex2(fmaf(x[2 * i], c, nbase)), p1 = ex2(fmaf(x[2 * i + 1], c, nbase));
-            sm[i & 3] += p0 + p1;
+            float a0, a1;
+            f2_unpack(f2_fma(f2_pack(x[2 * i], x[2 * i + 1]), c2, nb2), a0, a1);
+            const float p0 = ex2(a0), p1 = ex2(a1);
+            sm2[i & 1] = f2_add(sm2[i & 1], f2_pack(p0, p1));
             pk[i] = pack_bf16(p0, p1);
           }
+          float sm[4];
+          f2_unpack(sm2[0], sm[0], sm[1]);
+          f2_unpack(sm2[1], sm[2], sm[3]);
           // P #sc into its buffer: the PV product that last read it (#sc - 2)
           // completed before the previous tile's P was published
           tmem_st32(tl + kColP + m * 64 + pbuf * 32, pk);
