@@ -35,7 +35,7 @@ import torch  # noqa: E402
 # DRAM bytes (read + write) of one tree-attention launch on this workload, from
 # one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
 # source with the given sha256 prefix; another source reports null
-ATTN_TRAFFIC = {"f7b619d89bf865b0": 313165312}
+ATTN_TRAFFIC = {"516af6859f87a79b": 313298432}
 
 METRIC = "repair-verify steps/s at batch 32, block 16; tree-attn & vocab-scan HBM GB/s vs peak"
 WORKLOAD = "serve32"

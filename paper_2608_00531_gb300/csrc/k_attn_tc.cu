@@ -13,26 +13,35 @@
 // piece, and the CTA that completes the unit's last piece (a per-unit counter,
 // fence + atomic, no waiting) merges the pieces and writes the output.
 //
-// Roles (11 warps):
+// Roles (12 warps):
 //   warps 0-3 / 4-7   softmax of M tile 0 / 1: thread t owns row t = TMEM lane t
 //                     and writes its bf16 probabilities back into TMEM
 //   warp 8            TMA producer: Q rows (4-D box: d x group head x node),
 //                     64-key K and V tiles into 4-stage rings (128-byte
 //                     swizzle), page ids prefetched, boxes issued from
-//                     several lanes
-//   warps 9 / 10      MMA issuers (one lane each) of M tile 0 / 1:
-//                     S_m = Q_m K^T (M128 N64 K128) into TMEM S_m;
-//                     O_m += P_m V (A = P_m in TMEM, M128 N128 K64).
-//                     Issuing a tcgen05.mma costs the issuing thread about as
-//                     long as a 64-column product takes to run, so each M
-//                     tile has its own issuer.
+//                     several lanes.  A K tile is [d half][64 keys][64 d]
+//                     (K-major operand); a V tile is [16-key chunk][d half]
+//                     [16 keys][64 d], so that one 4 KiB box (both d halves
+//                     of 16 keys of one page) fills a chunk: a page costs one
+//                     V box instead of two, and fewer, larger boxes load faster
+//   warps 9 / 10      S issuers (one lane each) of M tile 0 / 1:
+//                     S_m = Q_m K^T (M128 N64 K128) into TMEM S_m
+//   warp 11           PV issuer (one lane) of both M tiles:
+//                     O_m += P_m V (A = P_m in TMEM, M128 N128 K64); it
+//                     releases the K/V stage after the tile's last product.
+//                     S is on the softmax's critical path and PV is not, so
+//                     an S product never queues behind a PV issue.  The
+//                     products of one group go out from one asm block with
+//                     constant descriptor steps, which keeps the issuing
+//                     lanes' instruction count low while the softmax warps
+//                     share their schedulers.
 // TMEM (512 columns): S[2] (2 x 64) | P[2][2] (4 x 32, bf16 pairs) | O[2]
 // (2 x 128).  The softmax releases S_m as soon as it has loaded it, so the
 // next tile's S product runs while this tile's exponentials are computed; P
 // is double-buffered so that it can be written while the previous PV product
-// still reads the other buffer.  The order of one issuer is
-//   S(0), S(1), PV(0), S(2), PV(1), ...
-// and a K/V ring stage is released when the PV product of its tile is done.
+// still reads the other buffer.  S(j + 1) is issued as soon as the softmax
+// has loaded S(j); PV(j) as soon as it has published P(j); a K/V ring stage
+// is released when the PV products of its tile are done.
 // The online softmax keeps a lazily updated row max (O is rescaled in TMEM only
 // when the max grows by more than 2^8).  Every mbarrier wait is bounded; on a
 // timeout the CTA raises CURE_DEVERR_TIMEOUT, drains and leaves.
@@ -53,12 +62,14 @@ constexpr int BM = kAttnRowsCta;  // 128 rows per M tile
 constexpr int BN = kAttnKeys;     // 64 keys per tile
 constexpr int D = kAttnD;         // 128
 constexpr int NS = 4;             // K and V ring stages
-constexpr int kThreads = 352;     // 11 warps
+constexpr int kThreads = 384;     // 12 warps
 constexpr uint32_t kTmemCols = 512;
 
 constexpr int kQHalf = BM * 64 * 2;   // 16 KiB: [128 rows][64 d]
 constexpr int kKVHalf = BN * 64 * 2;  // 8 KiB: [64 keys][64 d]
 constexpr int kTile = 2 * kKVHalf;    // one K or V tile (16 KiB)
+constexpr int kVChunk = 16 * D * 2;   // 4 KiB: V keys 16c..16c+15, both d halves
+constexpr int kVHalf = kVChunk / 2;   // 2 KiB: one d half of a V chunk
 constexpr int kOffQ = 0;                          // Q[m][half]
 constexpr int kOffK = kOffQ + 4 * kQHalf;         // K[stage]
 constexpr int kOffV = kOffK + NS * kTile;         // V[stage]
@@ -66,7 +77,7 @@ constexpr int kOffMisc = kOffV + NS * kTile;      // 196608
 enum {
   B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_VFULL = B_KFULL + NS, B_KVEMPTY = B_VFULL + NS,
   B_SFULL = B_KVEMPTY + NS, B_SFREE = B_SFULL + 2, B_PFULL = B_SFREE + 2, B_PVDONE = B_PFULL + 2,
-  B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 2
+  B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 3
 };
 constexpr int kOffTmemSlot = kOffMisc + 8 * kNumBars;
 constexpr int kOffAbort = kOffTmemSlot + 4;
@@ -79,6 +90,51 @@ constexpr uint32_t kColS = 0;    // S[m]:      columns m*64
 constexpr uint32_t kColP = 128;  // P[m][buf]: columns 128 + m*64 + buf*32
 constexpr uint32_t kColO = 256;  // O[m]:      columns 256 + m*128
 constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
+
+// One S product group, S_m = Q_m K^T over K = 128 (8 MMAs), in one asm
+// block: the descriptors step by constant adds (16-byte units: 32 bytes
+// within a 64-element half, a whole half of Q or K between ks = 3 and 4).
+__device__ __forceinline__ void mma_s_group(uint32_t d, uint64_t qd, uint64_t kd, uint32_t idesc) {
+  asm volatile(
+      "{\n\t.reg .pred pf, pt;\n\t.reg .b64 a, b;\n\t"
+      "setp.ne.b32 pf, %4, %4;\n\t"
+      "setp.eq.b32 pt, %4, %4;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, pf;\n\t"
+      "add.s64 a, %1, 2;\n\tadd.s64 b, %2, 2;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, 4;\n\tadd.s64 b, %2, 4;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, 6;\n\tadd.s64 b, %2, 6;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, %5;\n\tadd.s64 b, %2, %6;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, %5 + 2;\n\tadd.s64 b, %2, %6 + 2;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, %5 + 4;\n\tadd.s64 b, %2, %6 + 4;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
+      "add.s64 a, %1, %5 + 6;\n\tadd.s64 b, %2, %6 + 6;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t}\n" ::"r"(d),
+      "l"(qd), "l"(kd), "r"(idesc), "r"(0), "n"(kQHalf >> 4), "n"(kKVHalf >> 4)
+      : "memory");
+}
+// One PV product group, O_m (+)= P_m V over 64 keys (4 MMAs): A from TMEM
+// (8 columns of bf16 pairs per step), B stepping by one V chunk.
+__device__ __forceinline__ void mma_pv_group(uint32_t d, uint32_t pa, uint64_t vd, uint32_t idesc,
+                                             uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p0, pt;\n\t.reg .b64 b;\n\t.reg .b32 t;\n\t"
+      "setp.ne.b32 p0, %4, 0;\n\t"
+      "setp.eq.b32 pt, %4, %4;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p0;\n\t"
+      "add.u32 t, %1, 8;\n\tadd.s64 b, %2, %5;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t], b, %3, pt;\n\t"
+      "add.u32 t, %1, 16;\n\tadd.s64 b, %2, 2 * %5;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t], b, %3, pt;\n\t"
+      "add.u32 t, %1, 24;\n\tadd.s64 b, %2, 3 * %5;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [t], b, %3, pt;\n\t}\n" ::"r"(d),
+      "r"(pa), "l"(vd), "r"(idesc), "r"(accumulate), "n"(kVChunk >> 4)
+      : "memory");
+}
 
 struct Bar {
   uint32_t base;
@@ -179,6 +235,14 @@ __device__ __forceinline__ void named_sync_softmax() {  // warps 0-7
   asm volatile("bar.sync 1, 256;" ::: "memory");
 }
 
+__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1, int c2, int c3, int c4) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+      : "memory");
+}
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
                                             int c0, int c1, int c2, int c3) {
   asm volatile(
@@ -279,7 +343,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     for (int i = 0; i < NS; ++i) {
       mbar_init(bar(B_KFULL + i), 1);
       mbar_init(bar(B_VFULL + i), 1);
-      mbar_init(bar(B_KVEMPTY + i), 2);
+      mbar_init(bar(B_KVEMPTY + i), 1);
     }
     for (int m = 0; m < 2; ++m) {
       mbar_init(bar(B_SFULL + m), 1);
@@ -289,6 +353,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       mbar_init(bar(B_OFREE + m), 128);
       mbar_init(bar(B_DRAIN + m), 1);
     }
+    mbar_init(bar(B_DRAIN + 2), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -437,31 +502,54 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         // The boxes of one tile are issued by several lanes at once (one box
         // each): a single issuing thread sustains only a few boxes per
         // microsecond, and a paged tile is 2 * (64 / page_size) boxes.
-        auto issue = [&](uint32_t dst, uint32_t fb, const CUtensorMap* cmap, const CUtensorMap* tmap) {
+        auto page_of = [&](int p) {
+          int pgv = tpg[0];
+#pragma unroll
+          for (int q = 1; q < 8; ++q) pgv = (q == p) ? tpg[q] : pgv;
+          return pgv;
+        };
+        auto issue_k = [&](uint32_t dst, uint32_t fb) {
           const int hf = lane & 1, p = lane >> 1;
           if (t < s.nct) {
             if (A.kv.layout == 0) {
               if (lane < 2)
-                tma_load_3d(dst + hf * kKVHalf, cmap, fb, hf * 64, s.h, s.b * A.kv.max_len + t * BN);
+                tma_load_3d(dst + hf * kKVHalf, &tm_k, fb, hf * 64, s.h, s.b * A.kv.max_len + t * BN);
             } else if (p < ppt) {
-              int pgv = tpg[0];
-#pragma unroll
-              for (int q = 1; q < 8; ++q) pgv = (q == p) ? tpg[q] : pgv;
-              tma_load_3d(dst + hf * kKVHalf + p * ps * 128, cmap, fb, hf * 64, s.h, pgv * ps);
+              tma_load_3d(dst + hf * kKVHalf + p * ps * 128, &tm_k, fb, hf * 64, s.h, page_of(p) * ps);
             }
           } else if (lane < 2) {
-            tma_load_3d(dst + hf * kKVHalf, tmap, fb, hf * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
+            tma_load_3d(dst + hf * kKVHalf, &tm_tk, fb, hf * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
+          }
+        };
+        // V chunk c = keys 16c..16c+15 of the tile (lanes 0-3); with 8-token
+        // pages each page is two 1 KiB boxes, one per d half (lanes 0-15)
+        auto issue_v = [&](uint32_t dst, uint32_t fb) {
+          if (t < s.nct) {
+            if (A.kv.layout == 0) {
+              if (lane < 4)
+                tma_load_4d(dst + lane * kVChunk, &tm_v, fb, 0, s.b * A.kv.max_len + t * BN + 16 * lane, 0, s.h);
+            } else if (ps == 8) {
+              const int hf = lane & 1, p = lane >> 1;
+              if (p < 8)
+                tma_load_3d(dst + (p >> 1) * kVChunk + hf * kVHalf + (p & 1) * (kVHalf / 2), &tm_v, fb,
+                            hf * 64, s.h, page_of(p) * 8);
+            } else if (lane < 4) {
+              const int key = 16 * lane;  // page key / ps of the tile, row key % ps within it
+              tma_load_5d(dst + lane * kVChunk, &tm_v, fb, 0, key % ps, 0, s.h, page_of(key / ps));
+            }
+          } else if (lane < 4) {
+            tma_load_4d(dst + lane * kVChunk, &tm_tv, fb, 0, s.b * A.n_max + (t - s.nct) * BN + 16 * lane, 0, s.h);
           }
         };
         if (!wait_warp(bar(B_KVEMPTY + st), ph, abort_flag, A.err)) { ok = false; break; }
         if (lane == 0) mbar_arrive_expect_tx(bar(B_KFULL + st), kTile);
         __syncwarp();
-        issue(sb + kOffK + st * kTile, bar(B_KFULL + st), &tm_k, &tm_tk);
+        issue_k(sb + kOffK + st * kTile, bar(B_KFULL + st));
         __syncwarp();
         ++k_issued;
         if (lane == 0) mbar_arrive_expect_tx(bar(B_VFULL + st), kTile);
         __syncwarp();
-        issue(sb + kOffV + st * kTile, bar(B_VFULL + st), &tm_v, &tm_tv);
+        issue_v(sb + kOffV + st * kTile, bar(B_VFULL + st));
         __syncwarp();
         ++v_issued;
         ++gk;
@@ -475,13 +563,13 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         wait_bounded(bar(B_VFULL + i % NS), (i / NS) & 1u, abort_flag, A.err, false);
       if (qc > 0) wait_bounded(bar(B_QFULL), (qc - 1) & 1u, abort_flag, A.err, false);
     }
-  } else if (warp >= 9) {
-    // ================================================================ MMA issuers
-    // warp 9 + m issues the products of M tile m
+  } else if (warp == 9 || warp == 10) {
+    // ================================================================ S issuers
+    // warp 9 + m issues S_m = Q_m K^T as soon as the softmax has loaded the
+    // previous S_m and the tile's K has landed
     const int m = warp - 9;
     constexpr uint32_t idS = idesc_bf16_f32(BM, BN, false);
-    constexpr uint32_t idO = idesc_bf16_f32(BM, D, true);
-    uint32_t qc = 0, gk = 0, sc = 0, pc = 0, oc = 0;
+    uint32_t qc = 0, gk = 0, sc = 0;
     bool ok = true;
     for (long long g = g_begin; ok && g < g_end;) {
       const Seg s = sch.at(g, g_end);
@@ -492,39 +580,55 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       gk += (uint32_t)n;
       if (!wait_warp(bar(B_QFULL), qc & 1u, abort_flag, A.err)) { ok = false; break; }
       ++qc;
-      if (!(m == 0 || active1(s))) {
-        // an M tile without rows in this piece still releases every stage
-        // (after its copy was issued, so at most once per phase)
-        for (int j = 0; ok && j < n; ++j) {
-          const uint32_t gt = gk0 + (uint32_t)j;
-          if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
-          if (lane == 0) mbar_arrive(bar(B_KVEMPTY + gt % NS));
-          __syncwarp();
-        }
+      if (!(m == 0 || active1(s))) {  // no rows in this M tile: Q is free at once
         if (lane == 0) mbar_arrive(bar(B_QEMPTY));
         __syncwarp();
         continue;
       }
-      // PV of tile jp of this piece: P #pc from its buffer, V from the ring
-      auto issue_pv = [&](int jp) -> bool {
-        const uint32_t gt = gk0 + (uint32_t)jp;
+      const uint64_t qd = sdesc_sw128(sb + kOffQ + 2 * m * kQHalf, 16, 1024);
+      for (int j = 0; ok && j < n; ++j) {
+        const uint32_t gt = gk0 + (uint32_t)j;
+        if (sc > 0 && !wait_warp(bar(B_SFREE + m), (sc - 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+        if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+        tc_fence_after();
+        if (lane == 0) {
+          mma_s_group(tmem + kColS + m * 64, qd, sdesc_sw128(sb + kOffK + (gt % NS) * kTile, 16, 1024), idS);
+          mma_commit(bar(B_SFULL + m));
+          if (j == n - 1) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
+        }
+        __syncwarp();
+        ++sc;
+      }
+    }
+    if (lane == 0) mma_commit(bar(B_DRAIN + m));
+    __syncwarp();
+    wait_bounded(bar(B_DRAIN + m), 0, abort_flag, A.err, false);
+  } else if (warp == 11) {
+    // ================================================================ PV issuer
+    // O_m += P_m V for both M tiles as soon as the softmax has published P_m;
+    // the K/V stage is released after the tile's last PV product
+    constexpr uint32_t idO = idesc_bf16_f32(BM, D, true);
+    uint32_t gk = 0, pc0 = 0, pc1 = 0, oc0 = 0, oc1 = 0;
+    bool ok = true;
+    for (long long g = g_begin; ok && g < g_end;) {
+      const Seg s = sch.at(g, g_end);
+      g = s.next;
+      if (s.t1 <= s.t0) continue;
+      const int n = s.t1 - s.t0;
+      const uint32_t gk0 = gk;
+      gk += (uint32_t)n;
+      const bool two = active1(s);
+      auto issue_pv = [&](int m, uint32_t& pc, uint32_t& oc, int j, uint32_t gt) -> bool {
         if (!wait_warp(bar(B_PFULL + m), pc & 1u, abort_flag, A.err)) return false;
-        if (jp == 0) {  // O_m holds the previous piece until its epilogue has read it
+        if (j == 0) {  // O_m holds the previous piece until its epilogue has read it
           if (!wait_warp(bar(B_OFREE + m), (oc & 1u) ^ 1u, abort_flag, A.err)) return false;
           ++oc;
         }
-        if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) return false;
         tc_fence_after();
         if (lane == 0) {
-          const uint32_t va = sb + kOffV + (gt % NS) * kTile;
-          const uint32_t pa = tmem + kColP + m * 64 + (pc & 1u) * 32;
-#pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            mma_bf16_ts(tmem + kColO + m * 128, pa + ks * 8,
-                        sdesc_sw128(va + ks * 16 * 128, kKVHalf, 1024), idO,
-                        (jp > 0 || ks > 0) ? 1u : 0u);
+          mma_pv_group(tmem + kColO + m * 128, tmem + kColP + m * 64 + (pc & 1u) * 32,
+                       sdesc_sw128(sb + kOffV + (gt % NS) * kTile, kVHalf, 1024), idO, j > 0 ? 1u : 0u);
           mma_commit(bar(B_PVDONE + m));
-          mma_commit(bar(B_KVEMPTY + gt % NS));  // the tile's K and V are both consumed
         }
         __syncwarp();
         ++pc;
@@ -532,31 +636,15 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       };
       for (int j = 0; ok && j < n; ++j) {
         const uint32_t gt = gk0 + (uint32_t)j;
-        // S_m is rewritten once the softmax has loaded the previous S
-        if (sc > 0 && !wait_warp(bar(B_SFREE + m), (sc - 1) & 1u, abort_flag, A.err)) { ok = false; break; }
-        if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
-        tc_fence_after();
-        if (lane == 0) {
-          const uint32_t qa = sb + kOffQ + 2 * m * kQHalf, ka = sb + kOffK + (gt % NS) * kTile;
-#pragma unroll
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t oq = (ks >> 2) * kQHalf + (ks & 3) * 32;
-            const uint32_t okk = (ks >> 2) * kKVHalf + (ks & 3) * 32;
-            mma_bf16_ss(tmem + kColS + m * 64, sdesc_sw128(qa + oq, 16, 1024),
-                        sdesc_sw128(ka + okk, 16, 1024), idS, ks > 0 ? 1u : 0u);
-          }
-          mma_commit(bar(B_SFULL + m));
-          if (j == n - 1) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
-        }
+        if (!wait_warp(bar(B_VFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
+        if (!issue_pv(0, pc0, oc0, j, gt) || (two && !issue_pv(1, pc1, oc1, j, gt))) { ok = false; break; }
+        if (lane == 0) mma_commit(bar(B_KVEMPTY + gt % NS));  // the tile's K and V are consumed
         __syncwarp();
-        ++sc;
-        if (j > 0 && !issue_pv(j - 1)) { ok = false; break; }
       }
-      if (ok && !issue_pv(n - 1)) ok = false;
     }
-    if (lane == 0) mma_commit(bar(B_DRAIN + m));
+    if (lane == 0) mma_commit(bar(B_DRAIN + 2));
     __syncwarp();
-    wait_bounded(bar(B_DRAIN + m), 0, abort_flag, A.err, false);
+    wait_bounded(bar(B_DRAIN + 2), 0, abort_flag, A.err, false);
   } else {
     // ================================================================ softmax
     const int m = warp >> 2;   // M tile
@@ -684,7 +772,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             const int nch = (BN - valid) * 16;
             for (int q = row; q < nch; q += BM) {
               const int rr = valid + (q >> 4), hf = (q >> 3) & 1, cc = q & 7;
-              st_shared_v4(vb + hf * kKVHalf + rr * 128 + cc * 16, 0u, 0u, 0u, 0u);
+              st_shared_v4(vb + (rr >> 4) * kVChunk + hf * kVHalf + (rr & 15) * 128 + cc * 16, 0u, 0u, 0u, 0u);
             }
             fence_proxy_async_smem();
           }
@@ -880,6 +968,34 @@ bool make_kv_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv, int b
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// V rows [rows][Hkv][128] bf16 viewed as (d in half, row, d half, head);
+// boxes of 64 d x 16 rows x 2 halves: [half][16 rows][64 d], one 4 KiB chunk.
+bool make_v_rows_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {64, (cuuint64_t)rows, 2, (cuuint64_t)Hkv};
+  cuuint64_t strides[3] = {(cuuint64_t)Hkv * D * 2, 128, (cuuint64_t)D * 2};
+  cuuint32_t box[4] = {64, 16, 2, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Paged V [pages][ps][Hkv][128] bf16 viewed as (d in half, row in page, d
+// half, head, page); boxes as above: 16 rows of one page (ps >= 16).
+bool make_v_pages_map(CUtensorMap* m, const void* base, uint64_t pages, int ps, int Hkv) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[5] = {64, (cuuint64_t)ps, 2, (cuuint64_t)Hkv, (cuuint64_t)pages};
+  cuuint64_t strides[4] = {(cuuint64_t)Hkv * D * 2, 128, (cuuint64_t)D * 2, (cuuint64_t)ps * Hkv * D * 2};
+  cuuint32_t box[5] = {64, 16, 2, 1, 1};
+  cuuint32_t es[5] = {1, 1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // q [tokens][Hkv][G][128] bf16 viewed as (d, group head, kv head, token); boxes
 // of 64 d x G x 1 x npb tokens: the rows of one M tile, (node, g) packed.
 bool make_q_map(CUtensorMap* m, const void* base, uint64_t tokens, int Hkv, int G, int npb) {
@@ -913,14 +1029,16 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
   bool ok;
   if (A.kv.layout == 0) {
     const uint64_t rows = (uint64_t)A.batch * A.kv.max_len;
-    ok = make_kv_map(&mk, A.kc, rows, Hkv, BN) && make_kv_map(&mv, A.vc, rows, Hkv, BN);
+    ok = make_kv_map(&mk, A.kc, rows, Hkv, BN) && make_v_rows_map(&mv, A.vc, rows, Hkv);
   } else {
-    const uint64_t rows = (uint64_t)A.kv.num_pages * A.kv.page_size;
-    ok = make_kv_map(&mk, A.kc, rows, Hkv, A.kv.page_size) &&
-         make_kv_map(&mv, A.vc, rows, Hkv, A.kv.page_size);
+    const int ps = A.kv.page_size;
+    const uint64_t rows = (uint64_t)A.kv.num_pages * ps;
+    ok = make_kv_map(&mk, A.kc, rows, Hkv, ps) &&
+         (ps == 8 ? make_kv_map(&mv, A.vc, rows, Hkv, ps)
+                  : make_v_pages_map(&mv, A.vc, (uint64_t)A.kv.num_pages, ps, Hkv));
   }
   const uint64_t trows = (uint64_t)A.batch * A.n_max;
-  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_kv_map(&mtv, A.tv, trows, Hkv, BN) &&
+  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_v_rows_map(&mtv, A.tv, trows, Hkv) &&
        make_q_map(&mq, A.q, trows, Hkv, A.G, BM / A.G);
   if (!ok) return cudaErrorInvalidValue;
   // a fresh tag per launch makes the piece counters left in the workspace

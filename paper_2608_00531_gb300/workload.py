@@ -212,18 +212,19 @@ def cache_lengths(w: Workload, seed: Optional[int] = None, batch: Optional[int] 
     return rng.integers(w.len_lo, w.len_hi + 1, size=B).astype(np.int32)
 
 
-def pages_needed(cache_len: np.ndarray, block: int) -> np.ndarray:
+def pages_needed(cache_len: np.ndarray, block: int, page_size: int = PAGE_SIZE) -> np.ndarray:
     """Pages a sequence needs to hold its cache plus one block's worth of growth."""
-    return (cache_len.astype(np.int64) + block + 1 + PAGE_SIZE - 1) // PAGE_SIZE
+    return (cache_len.astype(np.int64) + block + 1 + page_size - 1) // page_size
 
 
-def block_table(cache_len: np.ndarray, block: int, seed: int) -> tuple[np.ndarray, int]:
+def block_table(cache_len: np.ndarray, block: int, seed: int,
+                page_size: int = PAGE_SIZE) -> tuple[np.ndarray, int]:
     """Shuffled physical page ids per sequence; -1 marks unused slots.
 
     Returns (table int32 [B][max_pages], number of physical pages).
     """
     rng = np.random.default_rng(seed + 271828)
-    need = pages_needed(cache_len, block)
+    need = pages_needed(cache_len, block, page_size)
     total = int(need.sum())
     perm = rng.permutation(total).astype(np.int32)
     maxp = int(need.max())

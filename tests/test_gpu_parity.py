@@ -163,7 +163,7 @@ def test_build_tree_random_params(cure, seed):
 
 
 # ------------------------------------------------------------------ attention
-def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0, branches=3):
+def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0, branches=3, ps=16):
     rng = np.random.default_rng(seed)
     k = max(2, branches)
     margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
@@ -177,9 +177,9 @@ def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0,
     tk = W.normal_bf16((B, N, Hkv, D), qk_std, rng)
     tv = W.normal_bf16((B, N, Hkv, D), v_std, rng)
     if paged:
-        table, npages = W.block_table(L, K, seed)
-        kc = W.normal_bf16((npages, 16, Hkv, D), qk_std, rng)
-        vc = W.normal_bf16((npages, 16, Hkv, D), v_std, rng)
+        table, npages = W.block_table(L, K, seed, ps)
+        kc = W.normal_bf16((npages, ps, Hkv, D), qk_std, rng)
+        vc = W.normal_bf16((npages, ps, Hkv, D), v_std, rng)
     else:
         table, npages = None, 0
         cap = int(L.max()) + K + 2
@@ -192,7 +192,7 @@ def _run_attn(c, t, q, tk, tv, kc, vc, L, table, npages, Hkv):
     B = q.shape[0]
     if table is not None:
         bt = torch.from_numpy(table).to(DEV)
-        kv = c.kv_desc(Hkv, 128, table.shape[1], bt, 16, npages)
+        kv = c.kv_desc(Hkv, 128, table.shape[1], bt, kc.shape[1], npages)
     else:
         kv = c.kv_desc(Hkv, 128, kc.shape[1])
     out = c.cure_tree_attn(q.to(DEV), tk.to(DEV), tv.to(DEV), kc.to(DEV), vc.to(DEV), kv,
@@ -229,6 +229,20 @@ def test_tree_attn_small(cure, paged, Hq, Hkv, qk_std, v_std):
     got = _run_attn(cure, t, q, tk, tv, kc, vc, L, table, npages, Hkv)
     ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
                            1.0 / math.sqrt(128), table, 16)
+    _cmp_attn(got, ref, t)
+
+
+@pytest.mark.parametrize("ps", [8, 32, 64])
+@pytest.mark.parametrize("Hq,Hkv", [(28, 4), (32, 8)])
+def test_tree_attn_page_sizes(cure, ps, Hq, Hkv):
+    """Pages of 8, 32 and 64 tokens: a 64-key tile spans 8, 2 or 1 pages (the
+    16-token pages of the other cases span 4); ragged lengths as above."""
+    lens = [0, 37, 700, 2100, 64, 1000]
+    t, q, tk, tv, kc, vc, L, table, npages = _attn_case(6, 8, 6, Hq, Hkv, lens, True, 1.0, 1.0,
+                                                         seed=40 + ps, ps=ps)
+    got = _run_attn(cure, t, q, tk, tv, kc, vc, L, table, npages, Hkv)
+    ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128), table, ps)
     _cmp_attn(got, ref, t)
 
 
@@ -355,8 +369,9 @@ def test_accept_random_trees_with_ids(cure, seed):
 
 
 # ------------------------------------------------------------------ resync
-@pytest.mark.parametrize("paged", [False, True])
+@pytest.mark.parametrize("paged", [0, 8, 16, 32, 64])
 def test_resync(cure, paged):
+    """paged: the page size in tokens, 0 for the contiguous layout."""
     rng = np.random.default_rng(21 + int(paged))
     B, K, budget, Hkv, D, layers = 5, 8, 6, 4, 128, 3
     margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
@@ -370,9 +385,9 @@ def test_resync(cure, paged):
     tk = W.normal_bf16((layers, B, N, Hkv, D), 1.0, rng)
     tv = W.normal_bf16((layers, B, N, Hkv, D), 1.0, rng)
     if paged:
-        table, npages = W.block_table(L, K, 5)
-        shape = (npages, 16, Hkv, D)
-        kv = cure.kv_desc(Hkv, D, table.shape[1], torch.from_numpy(table).to(DEV), 16, npages)
+        table, npages = W.block_table(L, K, 5, paged)
+        shape = (npages, paged, Hkv, D)
+        kv = cure.kv_desc(Hkv, D, table.shape[1], torch.from_numpy(table).to(DEV), paged, npages)
     else:
         table = None
         shape = (B, int(L.max()) + K + 1, Hkv, D)
@@ -388,7 +403,7 @@ def test_resync(cure, paged):
     ko = [_f64(x) for x in kcs]
     vo = [_f64(x) for x in vcs]
     o_rs = oracle.resync(ko, vo, _f64(tk), _f64(tv), o_acc["path_nodes"], o_acc["accept_len"],
-                         o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, 16)
+                         o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, paged or 16)
     for key in ("cache_len", "draft_valid_len", "replay_tokens", "n_replay"):
         assert np.array_equal(rs[key].cpu().numpy(), o_rs[key]), key
     for l in range(layers):
