@@ -19,11 +19,14 @@
 //   warp 8            TMA producer: Q rows (4-D box: d x group head x node),
 //                     64-key K and V tiles into 4-stage rings (128-byte
 //                     swizzle), page ids prefetched, boxes issued from
-//                     several lanes.  A K tile is [d half][64 keys][64 d]
-//                     (K-major operand); a V tile is [16-key chunk][d half]
-//                     [16 keys][64 d], so that one 4 KiB box (both d halves
-//                     of 16 keys of one page) fills a chunk: a page costs one
-//                     V box instead of two, and fewer, larger boxes load faster
+//                     several lanes.  A tile from a paged cache is
+//                     [8-key group][d half][8 keys][64 d] for K and V alike:
+//                     one box per page of one head (a 5-D map), 2 KiB apart
+//                     groups, so a 16-token page costs one 4 KiB box per
+//                     operand.  A producer warp sustains only so many boxes a
+//                     microsecond, so fewer, larger boxes load faster.  Tree
+//                     tiles and contiguous caches use [d half][64 keys][64 d]
+//                     for K and [16-key chunk][d half][16 keys][64 d] for V.
 //   warps 9 / 10      S issuers (one lane each) of M tile 0 / 1:
 //                     S_m = Q_m K^T (M128 N64 K128) into TMEM S_m
 //   warp 11           PV issuer (one lane) of both M tiles:
@@ -70,14 +73,18 @@ constexpr int kKVHalf = BN * 64 * 2;  // 8 KiB: [64 keys][64 d]
 constexpr int kTile = 2 * kKVHalf;    // one K or V tile (16 KiB)
 constexpr int kVChunk = 16 * D * 2;   // 4 KiB: V keys 16c..16c+15, both d halves
 constexpr int kVHalf = kVChunk / 2;   // 2 KiB: one d half of a V chunk
+// Tiles from a paged cache: [8-key group][d half][8 keys][64 d], one TMA box
+// per page (its ps / 8 groups, both halves); 8-key groups 2 KiB apart.
+constexpr int kPgGroup = 8 * D * 2;   // 2 KiB
+constexpr int kPgHalf = kPgGroup / 2; // 1 KiB
 constexpr int kOffQ = 0;                          // Q[m][half]
 constexpr int kOffK = kOffQ + 4 * kQHalf;         // K[stage]
 constexpr int kOffV = kOffK + NS * kTile;         // V[stage]
 constexpr int kOffMisc = kOffV + NS * kTile;      // 196608
 enum {
   B_QFULL = 0, B_QEMPTY = 1, B_KFULL = 2, B_VFULL = B_KFULL + NS, B_KVEMPTY = B_VFULL + NS,
-  B_SFULL = B_KVEMPTY + NS, B_SFREE = B_SFULL + 2, B_PFULL = B_SFREE + 2, B_PVDONE = B_PFULL + 2,
-  B_OFREE = B_PVDONE + 2, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 3
+  B_SFULL = B_KVEMPTY + NS, B_SFREE = B_SFULL + 2, B_PFULL = B_SFREE + 2, B_PVDONE = B_PFULL + 4,
+  B_OFREE = B_PVDONE + 4, B_DRAIN = B_OFREE + 2, kNumBars = B_DRAIN + 3
 };
 constexpr int kOffTmemSlot = kOffMisc + 8 * kNumBars;
 constexpr int kOffAbort = kOffTmemSlot + 4;
@@ -93,8 +100,8 @@ constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
 // One S product group, S_m = Q_m K^T over K = 128 (8 MMAs), in one asm
 // block: the descriptors step by constant adds (16-byte units: 32 bytes
-// within a 64-element half, a whole half of Q or K between ks = 3 and 4).
-__device__ __forceinline__ void mma_s_group(uint32_t d, uint64_t qd, uint64_t kd, uint32_t idesc) {
+// within a 64-element half); kd and kd2 describe the two d halves of K.
+__device__ __forceinline__ void mma_s_group(uint32_t d, uint64_t qd, uint64_t kd, uint64_t kd2, uint32_t idesc) {
   asm volatile(
       "{\n\t.reg .pred pf, pt;\n\t.reg .b64 a, b;\n\t"
       "setp.ne.b32 pf, %4, %4;\n\t"
@@ -106,15 +113,15 @@ __device__ __forceinline__ void mma_s_group(uint32_t d, uint64_t qd, uint64_t kd
       "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
       "add.s64 a, %1, 6;\n\tadd.s64 b, %2, 6;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
-      "add.s64 a, %1, %5;\n\tadd.s64 b, %2, %6;\n\t"
+      "add.s64 a, %1, %5;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, %6, %3, pt;\n\t"
+      "add.s64 a, %1, %5 + 2;\n\tadd.s64 b, %6, 2;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
-      "add.s64 a, %1, %5 + 2;\n\tadd.s64 b, %2, %6 + 2;\n\t"
+      "add.s64 a, %1, %5 + 4;\n\tadd.s64 b, %6, 4;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
-      "add.s64 a, %1, %5 + 4;\n\tadd.s64 b, %2, %6 + 4;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t"
-      "add.s64 a, %1, %5 + 6;\n\tadd.s64 b, %2, %6 + 6;\n\t"
+      "add.s64 a, %1, %5 + 6;\n\tadd.s64 b, %6, 6;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, pt;\n\t}\n" ::"r"(d),
-      "l"(qd), "l"(kd), "r"(idesc), "r"(0), "n"(kQHalf >> 4), "n"(kKVHalf >> 4)
+      "l"(qd), "l"(kd), "r"(idesc), "r"(0), "n"(kQHalf >> 4), "l"(kd2)
       : "memory");
 }
 // One PV product group, O_m (+)= P_m V over 64 keys (4 MMAs): A from TMEM
@@ -348,8 +355,10 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     for (int m = 0; m < 2; ++m) {
       mbar_init(bar(B_SFULL + m), 1);
       mbar_init(bar(B_SFREE + m), 128);
-      mbar_init(bar(B_PFULL + m), 128);
-      mbar_init(bar(B_PVDONE + m), 1);
+      mbar_init(bar(B_PFULL + 2 * m), 128);
+      mbar_init(bar(B_PFULL + 2 * m + 1), 128);
+      mbar_init(bar(B_PVDONE + 2 * m), 1);
+      mbar_init(bar(B_PVDONE + 2 * m + 1), 1);
       mbar_init(bar(B_OFREE + m), 128);
       mbar_init(bar(B_DRAIN + m), 1);
     }
@@ -508,34 +517,29 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           for (int q = 1; q < 8; ++q) pgv = (q == p) ? tpg[q] : pgv;
           return pgv;
         };
+        // A paged cache tile is one box per page (lane p: page p of the
+        // tile, ps * 256 bytes into the stage); a contiguous cache tile or a
+        // tree tile is two 64-key K boxes (one per d half) and four 16-key V
+        // chunks.
         auto issue_k = [&](uint32_t dst, uint32_t fb) {
-          const int hf = lane & 1, p = lane >> 1;
           if (t < s.nct) {
             if (A.kv.layout == 0) {
               if (lane < 2)
-                tma_load_3d(dst + hf * kKVHalf, &tm_k, fb, hf * 64, s.h, s.b * A.kv.max_len + t * BN);
-            } else if (p < ppt) {
-              tma_load_3d(dst + hf * kKVHalf + p * ps * 128, &tm_k, fb, hf * 64, s.h, page_of(p) * ps);
+                tma_load_3d(dst + lane * kKVHalf, &tm_k, fb, lane * 64, s.h, s.b * A.kv.max_len + t * BN);
+            } else if (lane < ppt) {
+              tma_load_5d(dst + lane * ps * 256, &tm_k, fb, 0, 0, 2 * s.h, 0, page_of(lane));
             }
           } else if (lane < 2) {
-            tma_load_3d(dst + hf * kKVHalf, &tm_tk, fb, hf * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
+            tma_load_3d(dst + lane * kKVHalf, &tm_tk, fb, lane * 64, s.h, s.b * A.n_max + (t - s.nct) * BN);
           }
         };
-        // V chunk c = keys 16c..16c+15 of the tile (lanes 0-3); with 8-token
-        // pages each page is two 1 KiB boxes, one per d half (lanes 0-15)
         auto issue_v = [&](uint32_t dst, uint32_t fb) {
           if (t < s.nct) {
             if (A.kv.layout == 0) {
               if (lane < 4)
                 tma_load_4d(dst + lane * kVChunk, &tm_v, fb, 0, s.b * A.kv.max_len + t * BN + 16 * lane, 0, s.h);
-            } else if (ps == 8) {
-              const int hf = lane & 1, p = lane >> 1;
-              if (p < 8)
-                tma_load_3d(dst + (p >> 1) * kVChunk + hf * kVHalf + (p & 1) * (kVHalf / 2), &tm_v, fb,
-                            hf * 64, s.h, page_of(p) * 8);
-            } else if (lane < 4) {
-              const int key = 16 * lane;  // page key / ps of the tile, row key % ps within it
-              tma_load_5d(dst + lane * kVChunk, &tm_v, fb, 0, key % ps, 0, s.h, page_of(key / ps));
+            } else if (lane < ppt) {
+              tma_load_5d(dst + lane * ps * 256, &tm_v, fb, 0, 0, 2 * s.h, 0, page_of(lane));
             }
           } else if (lane < 4) {
             tma_load_4d(dst + lane * kVChunk, &tm_tv, fb, 0, s.b * A.n_max + (t - s.nct) * BN + 16 * lane, 0, s.h);
@@ -592,7 +596,11 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         if (!wait_warp(bar(B_KFULL + gt % NS), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
         tc_fence_after();
         if (lane == 0) {
-          mma_s_group(tmem + kColS + m * 64, qd, sdesc_sw128(sb + kOffK + (gt % NS) * kTile, 16, 1024), idS);
+          // a paged cache tile interleaves the d halves per 8-key group
+          const bool pgd = A.kv.layout == 1 && s.t0 + j < s.nct;
+          const uint32_t ka = sb + kOffK + (gt % NS) * kTile;
+          const uint32_t sbo = pgd ? kPgGroup : 1024u, kh = pgd ? kPgHalf : kKVHalf;
+          mma_s_group(tmem + kColS + m * 64, qd, sdesc_sw128(ka, 16, sbo), sdesc_sw128(ka + kh, 16, sbo), idS);
           mma_commit(bar(B_SFULL + m));
           if (j == n - 1) mma_commit(bar(B_QEMPTY));  // the piece's last use of Q
         }
@@ -619,16 +627,21 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       gk += (uint32_t)n;
       const bool two = active1(s);
       auto issue_pv = [&](int m, uint32_t& pc, uint32_t& oc, int j, uint32_t gt) -> bool {
-        if (!wait_warp(bar(B_PFULL + m), pc & 1u, abort_flag, A.err)) return false;
+        if (!wait_warp(bar(B_PFULL + 2 * m + (pc & 1u)), (pc >> 1) & 1u, abort_flag, A.err)) return false;
         if (j == 0) {  // O_m holds the previous piece until its epilogue has read it
           if (!wait_warp(bar(B_OFREE + m), (oc & 1u) ^ 1u, abort_flag, A.err)) return false;
           ++oc;
         }
         tc_fence_after();
         if (lane == 0) {
+          // V as an MN-major operand: the d halves LBO apart, 8-key groups SBO
+          // apart; a K = 16 step is 4 KiB in both layouts
+          const bool pgd = A.kv.layout == 1 && s.t0 + j < s.nct;
           mma_pv_group(tmem + kColO + m * 128, tmem + kColP + m * 64 + (pc & 1u) * 32,
-                       sdesc_sw128(sb + kOffV + (gt % NS) * kTile, kVHalf, 1024), idO, j > 0 ? 1u : 0u);
-          mma_commit(bar(B_PVDONE + m));
+                       sdesc_sw128(sb + kOffV + (gt % NS) * kTile, pgd ? kPgHalf : kVHalf,
+                                   pgd ? kPgGroup : 1024u),
+                       idO, j > 0 ? 1u : 0u);
+          mma_commit(bar(B_PVDONE + 2 * m + (pc & 1u)));
         }
         __syncwarp();
         ++pc;
@@ -651,7 +664,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
     const int row = tid & 127; // row within the M tile = TMEM lane
     const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float c = A.scale_log2;
-    uint32_t sc = 0, pvc = 0, gk = 0;
+    uint32_t sc = 0, gk = 0;
     bool ok = true;
     for (long long g = g_begin; g < g_end;) {
       const Seg s = sch.at(g, g_end);
@@ -669,7 +682,8 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
         for (int jj = 0; jj < n; ++jj) {
           const int t = s.t0 + jj;
           if (!wait_warp(bar(B_SFULL + m), sc & 1u, abort_flag, A.err)) { ok = false; break; }
-          const uint32_t pbuf = sc & 1u;
+          const uint32_t tcur = sc;  // this M tile's tile count: P buffer tcur & 1
+          const uint32_t pbuf = tcur & 1u;
           ++sc;
           tc_fence_after();
           uint32_t u0[32], u1[32];
@@ -735,15 +749,21 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           float sm[4];
           f2_unpack(sm2[0], sm[0], sm[1]);
           f2_unpack(sm2[1], sm[2], sm[3]);
-          // P #sc into its buffer: the PV product that last read it (#sc - 2)
-          // completed before the previous tile's P was published
-          tmem_st32(tl + kColP + m * 64 + pbuf * 32, pk);
-          // O_m is stable once the previous PV product has completed
-          if (jj > 0) {
-            if (!wait_warp(bar(B_PVDONE + m), pvc & 1u, abort_flag, A.err)) { ok = false; break; }
-            ++pvc;
+          // P(t) goes into buffer t & 1 once PV(t - 2), which read it last, is
+          // done (each buffer has its own done barrier: PV(t) completes phase
+          // t >> 1 of barrier t & 1, and PV(t) cannot start before P(t) is
+          // published, so a wait is never two phases behind)
+          if (tcur >= 2) {
+            if (!wait_warp(bar(B_PVDONE + 2 * m + pbuf), ((tcur >> 1) & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
             tc_fence_after();
-            if (__any_sync(0xffffffffu, need)) {
+          }
+          tmem_st32(tl + kColP + m * 64 + pbuf * 32, pk);
+          // O_m is rescaled only once PV(t - 1) is done
+          if (jj > 0 && __any_sync(0xffffffffu, need)) {
+            const uint32_t tp = tcur - 1;
+            if (!wait_warp(bar(B_PVDONE + 2 * m + (tp & 1u)), (tp >> 1) & 1u, abort_flag, A.err)) { ok = false; break; }
+            tc_fence_after();
+            {
               const float alpha = need ? ex2(m_run - m_new) : 1.f;
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
@@ -770,19 +790,22 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             if (!wait_warp(bar(B_VFULL + st), (gt / NS) & 1u, abort_flag, A.err)) { ok = false; break; }
             const uint32_t vb = sb + kOffV + st * kTile;
             const int nch = (BN - valid) * 16;
+            const bool pgd = A.kv.layout == 1 && !tree;
             for (int q = row; q < nch; q += BM) {
               const int rr = valid + (q >> 4), hf = (q >> 3) & 1, cc = q & 7;
-              st_shared_v4(vb + (rr >> 4) * kVChunk + hf * kVHalf + (rr & 15) * 128 + cc * 16, 0u, 0u, 0u, 0u);
+              const uint32_t off = pgd ? (rr >> 3) * kPgGroup + hf * kPgHalf + (rr & 7) * 128
+                                       : (rr >> 4) * kVChunk + hf * kVHalf + (rr & 15) * 128;
+              st_shared_v4(vb + off + cc * 16, 0u, 0u, 0u, 0u);
             }
             fence_proxy_async_smem();
           }
           tmem_wait_st();
           tc_fence_before();
-          mbar_arrive(bar(B_PFULL + m));
+          mbar_arrive(bar(B_PFULL + 2 * m + pbuf));
         }
-        if (ok) {
-          if (!wait_warp(bar(B_PVDONE + m), pvc & 1u, abort_flag, A.err)) ok = false;
-          ++pvc;
+        if (ok) {  // O_m is final once the piece's last PV product is done
+          const uint32_t tl_ = sc - 1;
+          if (!wait_warp(bar(B_PVDONE + 2 * m + (tl_ & 1u)), (tl_ >> 1) & 1u, abort_flag, A.err)) ok = false;
         }
         if (ok) tc_fence_after();
       }
@@ -982,14 +1005,16 @@ bool make_v_rows_map(CUtensorMap* m, const void* base, uint64_t rows, int Hkv) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Paged V [pages][ps][Hkv][128] bf16 viewed as (d in half, row in page, d
-// half, head, page); boxes as above: 16 rows of one page (ps >= 16).
-bool make_v_pages_map(CUtensorMap* m, const void* base, uint64_t pages, int ps, int Hkv) {
+// Paged K or V [pages][ps][Hkv][128] bf16 viewed as (d in half, row in an
+// 8-row group, d half + 2 * head, group in page, page); one box is a whole
+// page of one head: [group][d half][8 rows][64 d], ps * 256 bytes.
+bool make_page_map(CUtensorMap* m, const void* base, uint64_t pages, int ps, int Hkv) {
   auto fn = encode_fn();
   if (!fn) return false;
-  cuuint64_t dims[5] = {64, (cuuint64_t)ps, 2, (cuuint64_t)Hkv, (cuuint64_t)pages};
-  cuuint64_t strides[4] = {(cuuint64_t)Hkv * D * 2, 128, (cuuint64_t)D * 2, (cuuint64_t)ps * Hkv * D * 2};
-  cuuint32_t box[5] = {64, 16, 2, 1, 1};
+  cuuint64_t dims[5] = {64, 8, 2 * (cuuint64_t)Hkv, (cuuint64_t)(ps / 8), (cuuint64_t)pages};
+  cuuint64_t strides[4] = {(cuuint64_t)Hkv * D * 2, 128, (cuuint64_t)8 * Hkv * D * 2,
+                           (cuuint64_t)ps * Hkv * D * 2};
+  cuuint32_t box[5] = {64, 8, 2, (cuuint32_t)(ps / 8), 1};
   cuuint32_t es[5] = {1, 1, 1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -1032,10 +1057,8 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
     ok = make_kv_map(&mk, A.kc, rows, Hkv, BN) && make_v_rows_map(&mv, A.vc, rows, Hkv);
   } else {
     const int ps = A.kv.page_size;
-    const uint64_t rows = (uint64_t)A.kv.num_pages * ps;
-    ok = make_kv_map(&mk, A.kc, rows, Hkv, ps) &&
-         (ps == 8 ? make_kv_map(&mv, A.vc, rows, Hkv, ps)
-                  : make_v_pages_map(&mv, A.vc, (uint64_t)A.kv.num_pages, ps, Hkv));
+    ok = make_page_map(&mk, A.kc, (uint64_t)A.kv.num_pages, ps, Hkv) &&
+         make_page_map(&mv, A.vc, (uint64_t)A.kv.num_pages, ps, Hkv);
   }
   const uint64_t trows = (uint64_t)A.batch * A.n_max;
   ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_v_rows_map(&mtv, A.tv, trows, Hkv) &&
