@@ -221,7 +221,9 @@ cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch,
  * repair path wins at divergence depth d (else L_b + a + 1), and
  * replay_tokens[b] (int32 [B][K+2]) = the path tokens at depths d..a followed by
  * the token after the path (only that token on branch-0 wins), then -1;
- * n_replay[b] its length.  cache_len_out may alias cache_len_in.
+ * n_replay[b] its length.  cache_len_out may alias cache_len_in; no other
+ * output may overlap an input (the copies and the replay list are written by
+ * one kernel, the lengths after it only when cache_len_out aliases).
  * k_caches, v_caches: HOST arrays of `layers` device pointers (layers <= 128).
  */
 cure_status cure_resync_kv(int32_t layers, void* const* k_caches, void* const* v_caches,
