@@ -316,6 +316,43 @@ def test_tree_attn_full_serve_layer_sampled(cure):
     _cmp_attn(got, ref, t, seqs)
 
 
+@pytest.mark.parametrize("name,budget", [("single8b", None), ("long64", None), ("sweep16", 64)])
+def test_tree_attn_config_layer_sampled(cure, name, budget):
+    """One layer at the other configurations' full shapes, contiguous caches:
+    single8b (1 x 4096, 32/8 heads), long64 (64 x 32768, 64/8 heads, depth-2
+    repairs, 49 nodes: two row groups per kv head) and sweep16 at R = 64 (16 x
+    8192, up to 97 nodes: two ancestor words).  The oracle checks two
+    sequences, on their own."""
+    w = W.WORKLOADS[name]
+    budget = w.budget if budget is None else budget
+    wt = w.replace(vocab=4096)  # the tree does not depend on the vocabulary
+    d, ids, margin = _tree_inputs(wt)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, budget, w.branches, w.repair_depth,
+                          d.redraft if w.repair_depth > 1 else None)
+    rng = np.random.default_rng(17)
+    N, D = 1 + w.block + budget, 128
+    q = W.normal_bf16((w.batch, N, w.heads_q, D), 1.0, rng)
+    tk = W.normal_bf16((w.batch, N, w.heads_kv, D), 1.0, rng)
+    tv = W.normal_bf16((w.batch, N, w.heads_kv, D), 1.0, rng)
+    cap = int(L.max())
+    g = torch.Generator(device=DEV).manual_seed(19)
+    kc = torch.randn(w.batch, cap, w.heads_kv, D, generator=g, device=DEV, dtype=torch.bfloat16)
+    vc = torch.randn(w.batch, cap, w.heads_kv, D, generator=g, device=DEV, dtype=torch.bfloat16)
+    kv = cure.kv_desc(w.heads_kv, D, cap)
+    out = cure.cure_tree_attn(q.to(DEV), tk.to(DEV), tv.to(DEV), kc, vc, kv, torch.from_numpy(L).to(DEV),
+                              torch.from_numpy(t["n_nodes"].astype(np.int32)).to(DEV),
+                              torch.from_numpy(t["anc"].view(np.int64)).to(DEV), 1.0 / math.sqrt(D))
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    got = out.float().cpu().numpy()
+    seqs = sorted({int(np.argmax(t["n_nodes"])), int(np.argmin(L))})
+    sub = {k_: v[seqs] for k_, v in t.items()}
+    ref = oracle.tree_attn(_f64(q)[seqs], _f64(tk)[seqs], _f64(tv)[seqs], _f64(kc[seqs].cpu()),
+                           _f64(vc[seqs].cpu()), L[seqs], sub["n_nodes"], sub["anc"], 1.0 / math.sqrt(D))
+    _cmp_attn(got[seqs], ref, sub)
+
+
 # ------------------------------------------------------------------ accept
 def _target_for(w, d, t, seed):
     truth = W.target_truth(w, d, seed)
