@@ -11,7 +11,8 @@ Stages and the passages they follow:
 
 * ``score_draft``  Sec. 3.3, Eq. (2) and Alg. 1 (draft scores and margin)
 * ``build_tree``   Sec. 3.1 Eq. (1) (budget), Sec. 3.3 (gate, ascending-margin
-                   order), Sec. 3.4 (tree construction, branch 0 anchored)
+                   order, Eq. (3) dynamic branch budget), Sec. 3.4 (tree
+                   construction, branch 0 anchored)
 * ``tree_attn``    Sec. 3.2 / 3.4 / 3.5 (single-pass Tree Attention)
 * ``accept``       Sec. 3.5 Eq. (4) with greedy decoding (Sec. 4.1)
 * ``resync``       Sec. 3.5 and Alg. 1 (cache resynchronisation)
@@ -27,6 +28,11 @@ notes of the repository):
   alternative that does not fit in the remaining budget R is skipped;
 * node 0 is the root (last committed token, position L), nodes 1..K are the
   draft chain, repair nodes follow in (position, rank, depth) order;
+* Eq. (3), when a margin scale s > 0 is given: b_i counts the alternatives of
+  UFP i (ranks 2..b_i + 1), with b_max = branches - 1 (the fixed budget's
+  alternatives) and b_min = branch_min; u_i, the product and the sum are
+  float32 operations, each rounded to nearest, and round() is half away from
+  zero;
 * the best path is the deepest accepted node, lowest node index on ties;
 * resync writes the path's rows (root included) into cache slots L..L+a and
   realigns the draft to L + divergence depth (or L + a + 1 on branch-0 wins).
@@ -89,14 +95,35 @@ def row_argmax(logits: np.ndarray) -> np.ndarray:
 # --------------------------------------------------------------------------
 # S2 + S3: UFP selection and tree construction (Sec. 3.1, 3.3, 3.4)
 # --------------------------------------------------------------------------
+def branch_budget(margin_f32: float, scale: float, b_min: int, b_max: int) -> int:
+    """Local branch budget of one UFP, Eq. (3) (Sec. 3.3, dynamic branching).
+
+    u = clip(1 - m / s, 0, 1) and b = clip(round(b_min + u (b_max - b_min)),
+    b_min, b_max): a confident position (m near s) keeps b_min alternatives,
+    a tied one (m = 0) gets b_max.  Each operation is a float32 operation
+    rounded to nearest (the precision the kernels hold the margin in); round()
+    takes halves away from zero.
+    """
+    f = np.float32
+    q = f(f(margin_f32) / f(scale))
+    u = f(f(1.0) - q)
+    u = f(min(max(u, f(0.0)), f(1.0)))
+    x = f(f(b_min) + f(u * f(b_max - b_min)))
+    r = math.floor(float(x) + 0.5)  # x >= 0: half away from zero
+    return int(min(max(r, b_min), b_max))
+
+
 def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
-                branches: int, repair_depth: int, max_ufp: int = 0):
+                branches: int, repair_depth: int, max_ufp: int = 0,
+                margin_scale: float = 0.0, branch_min: int = 1):
     """Budgeted ascending-margin selection of Uncertainty Focal Points.
 
     Sec. 3.3: positions with m_i < tau are UFPs, taken in ascending order of
-    m_i while the tree stays within the verifier budget (Eq. 1).  Returns the
-    admitted alternatives as a list of (position i, rank r) with r = 2..branches,
-    in admission order, and the UFP positions that received one.
+    m_i while the tree stays within the verifier budget (Eq. 1).  UFP i offers
+    the alternatives of ranks 2..branches, or, with a margin scale s > 0, the
+    b_i of ranks 2..b_i + 1 that Eq. (3) gives it (b_max = branches - 1).
+    Returns the admitted alternatives as a list of (position i, rank r), in
+    admission order, and the UFP positions that received one.
     """
     t32 = np.float32(tau)
     gated = [i for i in range(K) if np.float32(margin_f32[i]) < t32]
@@ -108,8 +135,11 @@ def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
     ufps = []
     for i in gated:
         cost = min(repair_depth, K - i)
+        nalt = branches - 1
+        if margin_scale > 0:
+            nalt = branch_budget(margin_f32[i], margin_scale, branch_min, branches - 1)
         took = False
-        for r in range(2, branches + 1):
+        for r in range(2, nalt + 2):
             if used + cost <= budget:
                 admitted.append((i, r))
                 used += cost
@@ -122,7 +152,7 @@ def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
 def build_tree(top_ids: np.ndarray, margin: np.ndarray, root_tok: np.ndarray,
                cache_len: np.ndarray, tau: float, budget: int, branches: int,
                repair_depth: int, redraft: Optional[np.ndarray] = None,
-               max_ufp: int = 0):
+               max_ufp: int = 0, margin_scale: float = 0.0, branch_min: int = 1):
     """Flattened repair tree per sequence (Sec. 3.4, Alg. 1 loop).
 
     Node 0: root (the last committed token) at depth 0, position L.
@@ -144,7 +174,8 @@ def build_tree(top_ids: np.ndarray, margin: np.ndarray, root_tok: np.ndarray,
     ufp_pos = np.full((B, K), -1, dtype=np.int64)
     n_ufp = np.zeros(B, dtype=np.int64)
     for b in range(B):
-        admitted, ufps = select_ufps(margin[b], tau, K, budget, branches, repair_depth, max_ufp)
+        admitted, ufps = select_ufps(margin[b], tau, K, budget, branches, repair_depth, max_ufp,
+                                     margin_scale, branch_min)
         n_ufp[b] = len(ufps)
         ufp_pos[b, :len(ufps)] = ufps
         nodes = [(int(root_tok[b]), -1, 0)]                 # (token, parent, depth)

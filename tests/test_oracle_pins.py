@@ -260,6 +260,100 @@ def test_tree_depth2_last_position_costs_one():
     assert t["depth"][0, 5:8].tolist() == [1, 2, 4]
 
 
+# ------------------------------------------------- Eq. (3) branch budget pins
+def test_branch_budget_closed_forms():
+    """Eq. (3) by hand at the paper's (b_min, b_max) = (1, 5).
+
+    With s = 8 every quotient m / s, every u = 1 - m / s and every
+    x = 1 + 4u below is exact in float32, so the expected b is the rounded
+    hand value; x = 1.5, 2.5, 3.5 and 4.5 pin the halves (away from zero:
+    half to even would give 2, 2, 4, 4).
+    """
+    bb = oracle.branch_budget
+    cases = [(0.0, 5),    # u = 1: a tied position gets b_max
+             (2.0, 4),    # u = 3/4: x = 4
+             (3.0, 4),    # u = 5/8: x = 3.5
+             (4.0, 3),    # u = 1/2: x = 3
+             (5.0, 3),    # u = 3/8: x = 2.5
+             (6.0, 2),    # u = 1/4: x = 2
+             (7.0, 2),    # u = 1/8: x = 1.5
+             (1.0, 5),    # u = 7/8: x = 4.5
+             (8.0, 1),    # u = 0: b_min
+             (12.0, 1)]   # m > s: u clipped to 0
+    for m, want in cases:
+        assert bb(np.float32(m), 8.0, 1, 5) == want, (m, want)
+    for m in (0.0, 0.3, 7.9, 100.0):          # b_min = b_max: constant
+        assert bb(np.float32(m), 1.0, 3, 3) == 3
+    assert bb(np.float32(1.0), 1.0, 0, 4) == 0    # b_min = 0 is reachable
+    assert bb(np.float32(0.0), 1.0, 0, 4) == 4
+    assert bb(np.float32(np.inf), 1.0, 1, 5) == 1  # rival at -inf: margin +inf
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_branch_budget_bounded_monotone_nearest(seed):
+    rng = np.random.default_rng(seed)
+    s = float(rng.choice([0.25, 0.8, 1.0, 2.5]))
+    b_min = int(rng.integers(0, 3))
+    b_max = b_min + int(rng.integers(0, 5))
+    ms = np.sort(rng.uniform(0.0, 2.0 * s, 400).astype(np.float32))
+    bs = [oracle.branch_budget(m, s, b_min, b_max) for m in ms]
+    assert all(b_min <= b <= b_max for b in bs)
+    assert all(x >= y for x, y in zip(bs, bs[1:]))      # more margin, fewer branches
+    for m, b in zip(ms, bs):                             # the nearest integer (exact arithmetic)
+        x = b_min + max(0.0, 1.0 - float(m) / s) * (b_max - b_min)
+        assert abs(b - x) <= 0.5 + 1e-5, (m, b, x)
+
+
+def _tree_dynamic_hand(budget):
+    K = 4
+    top = np.array([[[10 * i + r for r in range(6)] for i in range(K)]])
+    margin = np.array([[0.0, 0.5, 2.0, 0.75]], dtype=np.float32)
+    return oracle.build_tree(top, margin, np.array([7]), np.array([40]), 1.0, budget, 6, 1,
+                             margin_scale=1.0, branch_min=1)
+
+
+def test_tree_dynamic_budget_hand():
+    # tau = 1, s = 1, (b_min, b_max) = (1, 5): position 0 (m = 0) gets 5
+    # alternatives, position 1 (m = 0.5, x = 3) 3, position 3 (m = 0.75, x = 2)
+    # 2; position 2 (m = 2) is no UFP.  Nodes in (position, rank) order.
+    t = _tree_dynamic_hand(20)
+    assert t["n_nodes"][0] == 1 + 4 + 10
+    assert t["tok"][0, 5:15].tolist() == [1, 2, 3, 4, 5, 11, 12, 13, 31, 32]
+    assert t["parent"][0, 5:15].tolist() == [0] * 5 + [1] * 3 + [3] * 2
+    assert t["depth"][0, 5:15].tolist() == [1] * 5 + [2] * 3 + [4] * 2
+    assert t["ufp_pos"][0].tolist() == [0, 1, 3, -1] and t["n_ufp"][0] == 3
+    # budget 6: ascending margin admits position 0's five, then one of
+    # position 1's; position 3 no longer fits
+    t = _tree_dynamic_hand(6)
+    assert t["n_nodes"][0] == 1 + 4 + 6
+    assert t["tok"][0, 5:11].tolist() == [1, 2, 3, 4, 5, 11]
+    assert t["ufp_pos"][0].tolist() == [0, 1, -1, -1] and t["n_ufp"][0] == 2
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_tree_dynamic_budget_special_cases(seed):
+    top, margin, root, L, tau, budget, branches, d, redraft = _random_case(
+        seed, depth_rep=2 if seed % 2 else 1)
+    fixed = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft)
+    # b_min = b_max = branches - 1: every UFP keeps the fixed budget's alternatives
+    same = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft,
+                             margin_scale=float(1 + seed % 3), branch_min=branches - 1)
+    for key in fixed:
+        assert np.array_equal(fixed[key], same[key]), key
+    # m_i >= s for every position: Eq. (3) gives b_min everywhere (here 1)
+    one = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft,
+                            margin_scale=1e-6, branch_min=1)
+    ref1 = oracle.build_tree(top, margin, root, L, tau, budget, 2, d, redraft)
+    for b in range(top.shape[0]):
+        if (margin[b] > 0).all():
+            for key in ("n_nodes", "tok", "parent", "depth"):
+                assert np.array_equal(one[key][b], ref1[key][b]), key
+    # every tree with a dynamic budget keeps the invariants of a repair tree
+    dyn = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft,
+                            margin_scale=1.5, branch_min=1)
+    assert check_tree(dyn, top, margin, tau, budget, branches, d, L, redraft) == []
+
+
 # ---------------------------------------------------------------- S4 pins
 def _attn_case(seed, paged=False):
     rng = np.random.default_rng(seed)
