@@ -73,6 +73,10 @@ typedef struct {
                             the alternatives; 1..topk */
   int32_t repair_depth;  /* 1: alternative leaf; 2: alternative + its re-drafted successor */
   int32_t max_ufp;       /* 0 = no cap; else only the max_ufp lowest-margin UFPs are repaired */
+  float margin_scale;    /* s of Eq. (3); 0 = fixed budget (every UFP offers branches-1
+                            alternatives); > 0 and finite = dynamic budget (see cure_build_tree) */
+  int32_t branch_min;    /* b_min of Eq. (3), 0..branches-1 (the paper: 1); used when
+                            margin_scale > 0 */
 } cure_tree_params;
 
 /* KV-cache geometry (one layer). */
@@ -109,11 +113,20 @@ cure_status cure_score_draft(const void* logits, int32_t rows, int32_t vocab, in
  * Inputs:  top_ids int32 [B][K][topk] and margin float [B][K] (from stage 1),
  *          root_tok int32 [B] (last committed token), cache_len int32 [B] (L_b),
  *          redraft int32 [B][K][branches-1]: the successor token of each
- *          alternative when repair_depth == 2 (NULL otherwise).
+ *          alternative (rank r at index r-2) when repair_depth == 2 (NULL
+ *          otherwise).
  * Selection: positions with margin < tau, in ascending (margin, position)
  *   order; each alternative (i, r), r = 2..branches, costs min(repair_depth, K-i)
  *   nodes and is admitted while the repair nodes stay <= budget (an alternative
  *   that does not fit is skipped).
+ * Dynamic branch budget (Sec. 3.3, Eq. 3), when margin_scale s > 0: UFP i
+ *   offers the b_i alternatives of ranks 2..b_i+1 instead, with
+ *   u_i = clip(1 - m_i / s, 0, 1) and
+ *   b_i = clip(round(b_min + u_i (b_max - b_min)), b_min, b_max),
+ *   b_min = branch_min, b_max = branches - 1; the quotient, the difference, the
+ *   product and the sum are float32 operations rounded to nearest and round()
+ *   takes halves away from zero.  The paper's (b_min, b_max) = (1, 5) is
+ *   branch_min = 1, branches = 6 (topk >= 6).
  * Tree (n_max = 1 + K + budget nodes per sequence, W = ceil(n_max/64)):
  *   node 0 root (root_tok, depth 0); nodes 1..K branch 0 (top-1 ids, chained);
  *   then repair nodes in (i, r, depth) order: the rank-r id at position i as a

@@ -26,7 +26,8 @@ EXPORTS = ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_tree_a
 class TreeParams(C.Structure):
     _fields_ = [("batch", C.c_int32), ("block", C.c_int32), ("topk", C.c_int32),
                 ("tau", C.c_float), ("budget", C.c_int32), ("branches", C.c_int32),
-                ("repair_depth", C.c_int32), ("max_ufp", C.c_int32)]
+                ("repair_depth", C.c_int32), ("max_ufp", C.c_int32),
+                ("margin_scale", C.c_float), ("branch_min", C.c_int32)]
 
 
 class KVDesc(C.Structure):

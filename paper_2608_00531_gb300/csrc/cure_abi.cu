@@ -83,7 +83,7 @@ using namespace cure;
 
 extern "C" {
 
-int32_t cure_abi_version(void) { return 100; }
+int32_t cure_abi_version(void) { return 101; }
 
 const char* cure_status_string(cure_status s) {
   switch (s) {
@@ -116,7 +116,9 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
   if (!p) return CURE_ERR_INVALID_ARG;
   if (p->batch < 0 || p->block < 1 || p->block > 32 || p->topk < 2 || p->topk > 8 ||
       p->budget < 0 || p->branches < 1 || p->branches > p->topk ||
-      (p->repair_depth != 1 && p->repair_depth != 2) || p->max_ufp < 0)
+      (p->repair_depth != 1 && p->repair_depth != 2) || p->max_ufp < 0 ||
+      !(p->margin_scale >= 0.f && p->margin_scale <= FLT_MAX) ||
+      (p->margin_scale > 0.f && (p->branch_min < 0 || p->branch_min > p->branches - 1)))
     return CURE_ERR_INVALID_ARG;
   if (1 + p->block + p->budget > kMaxNodes) return CURE_ERR_UNSUPPORTED;
   if (p->batch == 0) return CURE_OK;

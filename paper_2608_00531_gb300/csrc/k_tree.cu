@@ -49,6 +49,7 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
   if (b >= p.batch) return;
   __shared__ int s_pos_by_rank[kWarpsPerCta][32];
   __shared__ int s_cnt[kWarpsPerCta][32];
+  __shared__ int s_nalt[kWarpsPerCta][32];
 
   const int K = p.block;
   const int k = p.topk;
@@ -70,8 +71,19 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
   if (p.max_ufp > 0 && rank >= p.max_ufp) gated = false;
   const unsigned gmask = __ballot_sync(kFull, gated);
   const int n_gated = __popc(gmask);
+  // alternatives this position offers: the fixed budget, or Eq. (3)'s b_i
+  // (u = clip(1 - m/s, 0, 1), b = clip(round(b_min + u (b_max - b_min))),
+  // each step a float32 operation rounded to nearest, halves away from zero)
+  int nalt_i = nalt;
+  if (p.margin_scale > 0.f) {
+    const int bmin = p.branch_min, bmax = nalt;
+    const float u = fminf(fmaxf(__fsub_rn(1.f, __fdiv_rn(m, p.margin_scale)), 0.f), 1.f);
+    const float x = __fadd_rn((float)bmin, __fmul_rn(u, (float)(bmax - bmin)));
+    nalt_i = min(max((int)roundf(x), bmin), bmax);
+  }
   if (gated) s_pos_by_rank[wib][rank] = lane;
   s_cnt[wib][lane] = 0;
+  s_nalt[wib][lane] = nalt_i;
   __syncwarp();
 
   // greedy admission in rank order; an alternative that does not fit is skipped
@@ -81,7 +93,8 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
       const int i = s_pos_by_rank[wib][q];
       const int cost = min(p.repair_depth, K - i);
       int c = 0;
-      for (int r = 0; r < nalt; ++r) {
+      const int na = s_nalt[wib][i];
+      for (int r = 0; r < na; ++r) {
         if (used + cost <= p.budget) {
           used += cost;
           ++c;

@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert lib.cure_abi_version() == 100
+    assert lib.cure_abi_version() == 101
     assert lib.cure_status_string(0) == b"ok"
     assert lib.cure_status_string(2) == b"workspace too small"
 
@@ -73,6 +73,13 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
     assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == 0
     p.batch, p.repair_depth = 1, 2      # depth-2 repairs need the re-drafted successors
     assert lib.cure_build_tree(C.byref(p), *([C.c_void_p(64)] * 5), null, *([C.c_void_p(64)] * 8), null) == 1
+    # Eq. (3) dynamic budget: s must be finite and >= 0; b_min within 0..branches-1
+    p.batch, p.repair_depth = 0, 1
+    for s, bmin, want in ((-1.0, 1, 1), (float("inf"), 1, 1), (float("nan"), 1, 1), (1.0, 3, 1),
+                          (1.0, -1, 1), (1.0, 2, 0), (1.0, 0, 0), (0.0, 7, 0)):
+        p.margin_scale, p.branch_min = s, bmin
+        assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == want, (s, bmin)
+    p.margin_scale, p.branch_min = 0.0, 1
     # attention: head_dim 64 unsupported, heads_q not a multiple of heads_kv
     kv = KVDesc(layout=0, heads_kv=4, head_dim=64, page_size=16, max_len=100, num_pages=0, block_table=None)
     assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 5

@@ -162,6 +162,58 @@ def test_build_tree_random_params(cure, seed):
     _cmp_tree(g, t)
 
 
+@pytest.mark.parametrize("seed", range(16))
+def test_build_tree_dynamic_budget_random(cure, seed):
+    """Eq. (3) dynamic branch budget: bit-exact against the oracle, including
+    margins on a grid where b_min + u (b_max - b_min) lands on halves."""
+    rng = np.random.default_rng(100 + seed)
+    B, K = int(rng.integers(1, 9)), int(rng.integers(1, 33))
+    k = int(rng.integers(2, 9))
+    branches = int(rng.integers(1, k + 1))
+    branch_min = int(rng.integers(0, branches))
+    depth = int(rng.integers(1, 3))
+    budget = int(rng.integers(0, 120))
+    scale = float(rng.choice([0.3, 0.8, 1.0, 2.5, 8.0]))
+    tau = float(rng.choice([0.5, 1.0, 3.0, 10.0]))
+    if seed % 2:
+        margin = (rng.integers(0, 40, size=(B, K)) * 0.25).astype(np.float32)
+    else:
+        margin = rng.exponential(1.0, size=(B, K)).astype(np.float32)
+    ids = rng.integers(0, 50000, size=(B, K, k))
+    root = rng.integers(0, 50000, size=B)
+    L = rng.integers(0, 1000, size=B)
+    redraft = rng.integers(0, 50000, size=(B, K, max(1, branches - 1)))
+    g = cure.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV), torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(root.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), tau, budget, branches, depth,
+                             torch.from_numpy(redraft.astype(np.int32)).to(DEV), 0,
+                             margin_scale=scale, branch_min=branch_min)
+    t = oracle.build_tree(ids, margin, root, L, tau, budget, branches, depth, redraft, 0,
+                          margin_scale=scale, branch_min=branch_min)
+    _cmp_tree(g, t)
+
+
+def test_build_tree_dynamic_budget_paper_setting(cure):
+    """The paper's dynamic branching, (b_min, b_max) = (1, 5), on the serving
+    shape's scores (top-6 candidates), s = tau."""
+    w = W.WORKLOADS["serve32"].replace(branches=6)
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    g = cure.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV), torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(d.root_tok.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), w.tau, w.budget, 6, 1, None, 0,
+                             margin_scale=w.tau, branch_min=1)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, 6, 1, None, 0,
+                          margin_scale=w.tau, branch_min=1)
+    _cmp_tree(g, t)
+    # the budget varies with the margin: some UFPs take more alternatives than others
+    counts = []
+    for b in range(w.batch):
+        par = t["parent"][b, 1 + w.block:int(t["n_nodes"][b])]
+        counts += [int((par == i).sum()) for i in set(par.tolist())]
+    assert len(set(counts)) > 1
+
+
 # ------------------------------------------------------------------ attention
 def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0, branches=3, ps=16):
     rng = np.random.default_rng(seed)
