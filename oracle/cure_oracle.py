@@ -33,6 +33,12 @@ notes of the repository):
   alternatives) and b_min = branch_min; u_i, the product and the sum are
   float32 operations, each rounded to nearest, and round() is half away from
   zero;
+* the structural caps of Sec. 3.3-3.4 bound repair branches only (branch 0
+  is never pruned): with a maximum depth, an alternative deeper than it is
+  not spawned and a successor deeper than it is dropped (the alternative then
+  costs one node, as at the last position); with a beam width, an
+  alternative is admitted only if every depth it occupies still holds fewer
+  nodes than the beam, the chain node included;
 * the best path is the deepest accepted node, lowest node index on ties;
 * resync writes the path's rows (root included) into cache slots L..L+a and
   realigns the draft to L + divergence depth (or L + a + 1 on branch-0 wins).
@@ -113,15 +119,28 @@ def branch_budget(margin_f32: float, scale: float, b_min: int, b_max: int) -> in
     return int(min(max(r, b_min), b_max))
 
 
+def repair_cost(i: int, K: int, repair_depth: int, max_depth: int = 0) -> int:
+    """Nodes one alternative at position i adds: itself (depth i + 1) and,
+    with depth-2 repairs, its successor (depth i + 2), within the block and
+    within the maximum depth (0 = none)."""
+    c = min(repair_depth, K - i)
+    if max_depth > 0:
+        c = min(c, max(0, max_depth - i))
+    return c
+
+
 def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
                 branches: int, repair_depth: int, max_ufp: int = 0,
-                margin_scale: float = 0.0, branch_min: int = 1):
+                margin_scale: float = 0.0, branch_min: int = 1,
+                max_depth: int = 0, beam: int = 0):
     """Budgeted ascending-margin selection of Uncertainty Focal Points.
 
     Sec. 3.3: positions with m_i < tau are UFPs, taken in ascending order of
     m_i while the tree stays within the verifier budget (Eq. 1).  UFP i offers
     the alternatives of ranks 2..branches, or, with a margin scale s > 0, the
     b_i of ranks 2..b_i + 1 that Eq. (3) gives it (b_max = branches - 1).
+    A maximum depth and a beam width (Sec. 3.3-3.4, 0 = none) bound where
+    alternatives may go: see ``repair_cost`` and the beam test below.
     Returns the admitted alternatives as a list of (position i, rank r), in
     admission order, and the UFP positions that received one.
     """
@@ -133,16 +152,23 @@ def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
     used = 0
     admitted = []
     ufps = []
+    width = [1] * (K + 2)          # nodes per depth: the root, then the chain
     for i in gated:
-        cost = min(repair_depth, K - i)
+        cost = repair_cost(i, K, repair_depth, max_depth)
+        if cost == 0:
+            continue
         nalt = branches - 1
         if margin_scale > 0:
             nalt = branch_budget(margin_f32[i], margin_scale, branch_min, branches - 1)
         took = False
         for r in range(2, nalt + 2):
-            if used + cost <= budget:
+            depths = range(i + 1, i + 1 + cost)
+            fits_beam = beam <= 0 or all(width[dd] < beam for dd in depths)
+            if used + cost <= budget and fits_beam:
                 admitted.append((i, r))
                 used += cost
+                for dd in depths:
+                    width[dd] += 1
                 took = True
         if took:
             ufps.append(i)
@@ -152,7 +178,8 @@ def select_ufps(margin_f32: Sequence[float], tau: float, K: int, budget: int,
 def build_tree(top_ids: np.ndarray, margin: np.ndarray, root_tok: np.ndarray,
                cache_len: np.ndarray, tau: float, budget: int, branches: int,
                repair_depth: int, redraft: Optional[np.ndarray] = None,
-               max_ufp: int = 0, margin_scale: float = 0.0, branch_min: int = 1):
+               max_ufp: int = 0, margin_scale: float = 0.0, branch_min: int = 1,
+               max_depth: int = 0, beam: int = 0):
     """Flattened repair tree per sequence (Sec. 3.4, Alg. 1 loop).
 
     Node 0: root (the last committed token) at depth 0, position L.
@@ -175,7 +202,7 @@ def build_tree(top_ids: np.ndarray, margin: np.ndarray, root_tok: np.ndarray,
     n_ufp = np.zeros(B, dtype=np.int64)
     for b in range(B):
         admitted, ufps = select_ufps(margin[b], tau, K, budget, branches, repair_depth, max_ufp,
-                                     margin_scale, branch_min)
+                                     margin_scale, branch_min, max_depth, beam)
         n_ufp[b] = len(ufps)
         ufp_pos[b, :len(ufps)] = ufps
         nodes = [(int(root_tok[b]), -1, 0)]                 # (token, parent, depth)
@@ -183,7 +210,7 @@ def build_tree(top_ids: np.ndarray, margin: np.ndarray, root_tok: np.ndarray,
             nodes.append((int(top_ids[b, i - 1, 0]), i - 1, i))
         for (i, r) in sorted(admitted):
             nodes.append((int(top_ids[b, i, r - 1]), i, i + 1))
-            if min(repair_depth, K - i) == 2:
+            if repair_cost(i, K, repair_depth, max_depth) == 2:
                 nodes.append((int(redraft[b, i, r - 2]), len(nodes) - 1, i + 2))
         assert len(nodes) <= n_max
         n_nodes[b] = len(nodes)

@@ -354,6 +354,74 @@ def test_tree_dynamic_budget_special_cases(seed):
     assert check_tree(dyn, top, margin, tau, budget, branches, d, L, redraft) == []
 
 
+# --------------------------------------- structural caps (depth, beam) pins
+def _caps_hand(**kw):
+    K = 4
+    top = np.array([[[100 * i + r for r in range(3)] for i in range(K)]])
+    margin = np.full((1, K), 0.1, dtype=np.float32)       # every position a UFP, ties by position
+    redraft = np.array([[[900 + 10 * i + a for a in range(2)] for i in range(K)]])
+    d = kw.pop("d", 1)
+    return oracle.build_tree(top, margin, np.array([5]), np.array([60]), 1.0, 40, 3, d, redraft, **kw)
+
+
+def test_tree_caps_hand():
+    # no caps: two alternatives at each of the four positions
+    assert _caps_hand()["n_nodes"][0] == 5 + 8
+    # beam 1: the chain fills every depth, so nothing is added
+    t = _caps_hand(beam=1)
+    assert t["n_nodes"][0] == 5 and t["n_ufp"][0] == 0
+    # beam 2: one alternative per depth, the rank-2 one (ranks are tried in order)
+    t = _caps_hand(beam=2)
+    assert t["n_nodes"][0] == 5 + 4
+    assert t["tok"][0, 5:9].tolist() == [1, 101, 201, 301]
+    # beam 3: everything fits again
+    assert _caps_hand(beam=3)["n_nodes"][0] == 5 + 8
+    # maximum depth 2: alternatives only at positions 0 and 1 (depths 1 and 2)
+    t = _caps_hand(max_depth=2)
+    assert t["n_nodes"][0] == 5 + 4
+    assert t["parent"][0, 5:9].tolist() == [0, 0, 1, 1]
+    assert t["ufp_pos"][0].tolist() == [0, 1, -1, -1]
+    # depth-2 repairs under maximum depth 2: position 0 keeps its successors
+    # (depths 1, 2); position 1's successors (depth 3) are dropped
+    t = _caps_hand(d=2, max_depth=2)
+    assert t["n_nodes"][0] == 5 + 6
+    assert t["tok"][0, 5:11].tolist() == [1, 900, 2, 901, 101, 102]
+    assert t["parent"][0, 5:11].tolist() == [0, 5, 0, 7, 1, 1]
+    assert t["depth"][0, 5:11].tolist() == [1, 2, 1, 2, 2, 2]
+    # depth-2 repairs under beam 2: position 0's first alternative and its
+    # successor take depths 1 and 2, so position 1 (depth 2) finds no room;
+    # position 2 fits (depths 3, 4); position 3 (depth 4) does not
+    t = _caps_hand(d=2, beam=2)
+    assert t["tok"][0, 5:].tolist()[:4] == [1, 900, 201, 920]
+    assert t["n_nodes"][0] == 5 + 4
+    assert t["ufp_pos"][0].tolist() == [0, 2, -1, -1]
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_tree_caps_invariants_and_no_op_values(seed):
+    depth_rep = 2 if seed % 2 else 1
+    top, margin, root, L, tau, budget, branches, d, redraft = _random_case(seed, depth_rep=depth_rep)
+    K = top.shape[1]
+    base = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft)
+    # caps that cannot bind change nothing
+    wide = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft,
+                             max_depth=K, beam=1 + 2 * branches)
+    for key in base:
+        assert np.array_equal(base[key], wide[key]), key
+    # binding caps: no repair node past the maximum depth, no depth wider
+    # than the beam, branch 0 intact
+    rng = np.random.default_rng(seed)
+    md, bw = int(rng.integers(1, K + 1)), int(rng.integers(1, 4))
+    t = oracle.build_tree(top, margin, root, L, tau, budget, branches, d, redraft, max_depth=md, beam=bw)
+    for b in range(top.shape[0]):
+        n = int(t["n_nodes"][b])
+        dep = t["depth"][b, :n]
+        assert (dep[1 + K:] <= md).all()
+        assert np.bincount(dep, minlength=K + 2).max() <= max(bw, 1)
+        assert t["tok"][b, 1:K + 1].tolist() == top[b, :, 0].tolist()
+        assert n <= 1 + K + budget
+
+
 # ---------------------------------------------------------------- S4 pins
 def _attn_case(seed, paged=False):
     rng = np.random.default_rng(seed)
