@@ -77,6 +77,8 @@ typedef struct {
                             alternatives); > 0 and finite = dynamic budget (see cure_build_tree) */
   int32_t branch_min;    /* b_min of Eq. (3), 0..branches-1 (the paper: 1); used when
                             margin_scale > 0 */
+  int32_t max_depth;     /* 0 = none; else no repair node deeper than max_depth (the paper: 15) */
+  int32_t beam;          /* 0 = none; else at most `beam` nodes at any depth (the paper: 5) */
 } cure_tree_params;
 
 /* KV-cache geometry (one layer). */
@@ -127,6 +129,12 @@ cure_status cure_score_draft(const void* logits, int32_t rows, int32_t vocab, in
  *   product and the sum are float32 operations rounded to nearest and round()
  *   takes halves away from zero.  The paper's (b_min, b_max) = (1, 5) is
  *   branch_min = 1, branches = 6 (topk >= 6).
+ * Structural caps (Sec. 3.3, 3.4; repair branches only, branch 0 is never
+ *   pruned): with max_depth > 0 an alternative at depth i+1 > max_depth is not
+ *   spawned and a successor at depth i+2 > max_depth is dropped (the
+ *   alternative then costs one node); with beam > 0 an alternative is admitted
+ *   only while every depth it occupies holds fewer than `beam` nodes, the chain
+ *   node included (one that does not fit is skipped, like the budget).
  * Tree (n_max = 1 + K + budget nodes per sequence, W = ceil(n_max/64)):
  *   node 0 root (root_tok, depth 0); nodes 1..K branch 0 (top-1 ids, chained);
  *   then repair nodes in (i, r, depth) order: the rank-r id at position i as a

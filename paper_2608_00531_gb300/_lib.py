@@ -27,7 +27,8 @@ class TreeParams(C.Structure):
     _fields_ = [("batch", C.c_int32), ("block", C.c_int32), ("topk", C.c_int32),
                 ("tau", C.c_float), ("budget", C.c_int32), ("branches", C.c_int32),
                 ("repair_depth", C.c_int32), ("max_ufp", C.c_int32),
-                ("margin_scale", C.c_float), ("branch_min", C.c_int32)]
+                ("margin_scale", C.c_float), ("branch_min", C.c_int32),
+                ("max_depth", C.c_int32), ("beam", C.c_int32)]
 
 
 class KVDesc(C.Structure):

@@ -83,7 +83,7 @@ using namespace cure;
 
 extern "C" {
 
-int32_t cure_abi_version(void) { return 101; }
+int32_t cure_abi_version(void) { return 102; }
 
 const char* cure_status_string(cure_status s) {
   switch (s) {
@@ -118,7 +118,8 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
       p->budget < 0 || p->branches < 1 || p->branches > p->topk ||
       (p->repair_depth != 1 && p->repair_depth != 2) || p->max_ufp < 0 ||
       !(p->margin_scale >= 0.f && p->margin_scale <= FLT_MAX) ||
-      (p->margin_scale > 0.f && (p->branch_min < 0 || p->branch_min > p->branches - 1)))
+      (p->margin_scale > 0.f && (p->branch_min < 0 || p->branch_min > p->branches - 1)) ||
+      p->max_depth < 0 || p->beam < 0)
     return CURE_ERR_INVALID_ARG;
   if (1 + p->block + p->budget > kMaxNodes) return CURE_ERR_UNSUPPORTED;
   if (p->batch == 0) return CURE_OK;

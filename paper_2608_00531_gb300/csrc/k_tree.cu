@@ -34,6 +34,15 @@ __device__ __forceinline__ void anc_prefix(uint64_t* dst, int W, int upto) {
   }
 }
 
+// Nodes one alternative at position i adds: itself (depth i + 1) and, with
+// depth-2 repairs, its successor (depth i + 2), within the block and within
+// the maximum depth (0 = none).
+__device__ __forceinline__ int repair_cost(int i, int K, int repair_depth, int max_depth) {
+  int c = min(repair_depth, K - i);
+  if (max_depth > 0) c = min(c, max(0, max_depth - i));
+  return c;
+}
+
 __global__ void __launch_bounds__(32 * kWarpsPerCta)
 build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
                   const float* __restrict__ margin, const int32_t* __restrict__ root_tok,
@@ -50,6 +59,7 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
   __shared__ int s_pos_by_rank[kWarpsPerCta][32];
   __shared__ int s_cnt[kWarpsPerCta][32];
   __shared__ int s_nalt[kWarpsPerCta][32];
+  __shared__ int s_width[kWarpsPerCta][34];  // nodes per depth 0..K+1 during admission
 
   const int K = p.block;
   const int k = p.topk;
@@ -84,19 +94,26 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
   if (gated) s_pos_by_rank[wib][rank] = lane;
   s_cnt[wib][lane] = 0;
   s_nalt[wib][lane] = nalt_i;
+  s_width[wib][lane] = 1;  // the root at depth 0, the chain node at depths 1..K
+  if (lane < 2) s_width[wib][32 + lane] = 1;
   __syncwarp();
 
-  // greedy admission in rank order; an alternative that does not fit is skipped
+  // greedy admission in rank order; an alternative that does not fit (the
+  // budget, or with a beam width a full depth) is skipped
   if (lane == 0) {
     int used = 0;
     for (int q = 0; q < n_gated; ++q) {
       const int i = s_pos_by_rank[wib][q];
-      const int cost = min(p.repair_depth, K - i);
+      const int cost = repair_cost(i, K, p.repair_depth, p.max_depth);
       int c = 0;
       const int na = s_nalt[wib][i];
-      for (int r = 0; r < na; ++r) {
-        if (used + cost <= p.budget) {
+      for (int r = 0; r < na && cost > 0; ++r) {
+        bool fits = used + cost <= p.budget;
+        if (p.beam > 0)
+          for (int dd = i + 1; dd <= i + cost; ++dd) fits = fits && s_width[wib][dd] < p.beam;
+        if (fits) {
           used += cost;
+          for (int dd = i + 1; dd <= i + cost; ++dd) ++s_width[wib][dd];
           ++c;
         }
       }
@@ -107,7 +124,7 @@ build_tree_kernel(cure_tree_params p, const int32_t* __restrict__ top_ids,
 
   // ---- S3: nodes in canonical (position, rank, depth) order
   const int cnt = valid ? s_cnt[wib][lane] : 0;
-  const int cost = valid ? min(p.repair_depth, K - lane) : 0;
+  const int cost = valid ? repair_cost(lane, K, p.repair_depth, p.max_depth) : 0;
   const int mine = cnt * cost;
   const int off = warp_excl_scan(mine, lane);
   const int total_rep = __shfl_sync(kFull, off + mine, 31);

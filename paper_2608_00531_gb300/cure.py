@@ -74,23 +74,25 @@ def cure_score_draft(logits: torch.Tensor, topk: int, *, out=None, stream=None):
 
 
 def tree_params(batch, block, topk, tau, budget, branches, repair_depth=1, max_ufp=0,
-                margin_scale=0.0, branch_min=1) -> TreeParams:
+                margin_scale=0.0, branch_min=1, max_depth=0, beam=0) -> TreeParams:
     p = TreeParams()
     p.batch, p.block, p.topk, p.tau = batch, block, topk, float(tau)
     p.budget, p.branches, p.repair_depth, p.max_ufp = budget, branches, repair_depth, max_ufp
     p.margin_scale, p.branch_min = float(margin_scale), branch_min
+    p.max_depth, p.beam = max_depth, beam
     return p
 
 
 def cure_build_tree(top_ids: torch.Tensor, margin: torch.Tensor, root_tok: torch.Tensor,
                     cache_len: torch.Tensor, tau: float, budget: int, branches: int,
                     repair_depth: int = 1, redraft: Optional[torch.Tensor] = None,
-                    max_ufp: int = 0, margin_scale: float = 0.0, branch_min: int = 1, *,
-                    out=None, stream=None) -> dict:
+                    max_ufp: int = 0, margin_scale: float = 0.0, branch_min: int = 1,
+                    max_depth: int = 0, beam: int = 0, *, out=None, stream=None) -> dict:
     """Stages 2+3 (Sec. 3.1 Eq. 1, Sec. 3.3, Sec. 3.4): the flattened repair tree.
 
     margin_scale > 0 turns on the dynamic branch budget of Eq. (3): UFP i then
-    offers b_i alternatives, from branch_min up to branches - 1."""
+    offers b_i alternatives, from branch_min up to branches - 1.  max_depth and
+    beam (0 = none) are the structural caps on repair branches (Sec. 3.3-3.4)."""
     _need(top_ids, torch.int32, "top_ids")
     _need(margin, torch.float32, "margin")
     B, K, k = top_ids.shape
@@ -106,7 +108,8 @@ def cure_build_tree(top_ids: torch.Tensor, margin: torch.Tensor, root_tok: torch
                    anc=torch.empty(B, n_max, W, dtype=torch.int64, device=dev),
                    ufp_pos=torch.empty(B, K, dtype=torch.int32, device=dev),
                    n_ufp=torch.empty(B, dtype=torch.int32, device=dev))
-    p = tree_params(B, K, k, tau, budget, branches, repair_depth, max_ufp, margin_scale, branch_min)
+    p = tree_params(B, K, k, tau, budget, branches, repair_depth, max_ufp, margin_scale, branch_min,
+                    max_depth, beam)
     lib = _lib.load()
     check("cure_build_tree", lib.cure_build_tree(
         C.byref(p), _p(top_ids), _p(margin), _p(root_tok), _p(cache_len), _p(redraft),

@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert lib.cure_abi_version() == 101
+    assert lib.cure_abi_version() == 102
     assert lib.cure_status_string(0) == b"ok"
     assert lib.cure_status_string(2) == b"workspace too small"
 
@@ -80,6 +80,10 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
         p.margin_scale, p.branch_min = s, bmin
         assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == want, (s, bmin)
     p.margin_scale, p.branch_min = 0.0, 1
+    for md, bw, want in ((-1, 0, 1), (0, -2, 1), (15, 5, 0), (0, 0, 0)):   # caps: >= 0
+        p.max_depth, p.beam = md, bw
+        assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == want, (md, bw)
+    p.max_depth, p.beam = 0, 0
     # attention: head_dim 64 unsupported, heads_q not a multiple of heads_kv
     kv = KVDesc(layout=0, heads_kv=4, head_dim=64, page_size=16, max_len=100, num_pages=0, block_table=None)
     assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 5

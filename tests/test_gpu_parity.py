@@ -214,6 +214,52 @@ def test_build_tree_dynamic_budget_paper_setting(cure):
     assert len(set(counts)) > 1
 
 
+@pytest.mark.parametrize("seed", range(16))
+def test_build_tree_caps_random(cure, seed):
+    """Maximum repair depth and beam width (with and without Eq. (3)),
+    bit-exact against the oracle."""
+    rng = np.random.default_rng(300 + seed)
+    B, K = int(rng.integers(1, 9)), int(rng.integers(1, 33))
+    k = int(rng.integers(2, 9))
+    branches = int(rng.integers(1, k + 1))
+    depth = int(rng.integers(1, 3))
+    budget = int(rng.integers(0, 120))
+    tau = float(rng.choice([0.5, 1.0, 3.0]))
+    max_depth = int(rng.choice([0, 1, 2, K // 2 + 1, K]))
+    beam = int(rng.choice([0, 1, 2, 3, 5]))
+    scale = float(rng.choice([0.0, 1.0]))
+    branch_min = int(rng.integers(0, branches)) if scale > 0 else 1
+    margin = (rng.integers(0, 16, size=(B, K)) * 0.25).astype(np.float32)
+    ids = rng.integers(0, 50000, size=(B, K, k))
+    root = rng.integers(0, 50000, size=B)
+    L = rng.integers(0, 1000, size=B)
+    redraft = rng.integers(0, 50000, size=(B, K, max(1, branches - 1)))
+    g = cure.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV), torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(root.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), tau, budget, branches, depth,
+                             torch.from_numpy(redraft.astype(np.int32)).to(DEV), 0,
+                             margin_scale=scale, branch_min=branch_min, max_depth=max_depth, beam=beam)
+    t = oracle.build_tree(ids, margin, root, L, tau, budget, branches, depth, redraft, 0,
+                          margin_scale=scale, branch_min=branch_min, max_depth=max_depth, beam=beam)
+    _cmp_tree(g, t)
+
+
+def test_build_tree_paper_primary_configuration(cure):
+    """The paper's primary configuration on the serving shape's top-6 scores:
+    tau = 1.0, at most one repaired position per block, up to 5 alternatives
+    (Eq. (3) with (b_min, b_max) = (1, 5), s = tau), maximum depth 15, beam 5."""
+    w = W.WORKLOADS["serve32"].replace(branches=6)
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    kw = dict(margin_scale=1.0, branch_min=1, max_depth=15, beam=5)
+    g = cure.cure_build_tree(torch.from_numpy(ids.astype(np.int32)).to(DEV), torch.from_numpy(margin).to(DEV),
+                             torch.from_numpy(d.root_tok.astype(np.int32)).to(DEV),
+                             torch.from_numpy(L.astype(np.int32)).to(DEV), 1.0, w.budget, 6, 1, None, 1, **kw)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, 1.0, w.budget, 6, 1, None, 1, **kw)
+    _cmp_tree(g, t)
+    assert (t["n_ufp"] <= 1).all() and (t["n_nodes"] <= 1 + w.block + 5).all()
+
+
 # ------------------------------------------------------------------ attention
 def _attn_case(B, K, budget, Hq, Hkv, lens, paged, qk_std, v_std, seed, tau=1.0, branches=3, ps=16):
     rng = np.random.default_rng(seed)
