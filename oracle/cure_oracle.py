@@ -41,7 +41,11 @@ notes of the repository):
   nodes than the beam, the chain node included;
 * the best path is the deepest accepted node, lowest node index on ties;
 * resync writes the path's rows (root included) into cache slots L..L+a and
-  realigns the draft to L + divergence depth (or L + a + 1 on branch-0 wins).
+  realigns the draft to L + divergence depth (or L + a + 1 on branch-0 wins);
+* in the in-place layout (the tree's K/V rows written by the target straight
+  into the cache) node j's row is cache slot L + j; attention and resync then
+  read the tree rows from there, and the result is the same as with separate
+  tree tensors holding those rows.
 
 Parity status: every function is pinned by tests that do not re-use its code
 (closed forms, brute force, textbook routines, invariants); see
@@ -255,7 +259,19 @@ def cache_rows(cache: np.ndarray, b: int, length: int, block_table: Optional[np.
     return np.stack(rows) if rows else np.zeros((0,) + cache.shape[2:])
 
 
-def tree_attn(q: np.ndarray, tree_k: np.ndarray, tree_v: np.ndarray,
+def tree_rows_in_cache(cache: np.ndarray, cache_len: np.ndarray, n_nodes: np.ndarray, N: int,
+                       block_table: Optional[np.ndarray], page_size: int) -> np.ndarray:
+    """The in-place layout's tree rows as [B][N][Hkv][D]: node j of sequence b
+    is cache slot L_b + j (rows past n_b stay zero)."""
+    B = len(cache_len)
+    out = np.zeros((B, N) + cache.shape[2:], dtype=cache.dtype)
+    for b in range(B):
+        L, n = int(cache_len[b]), int(n_nodes[b])
+        out[b, :n] = cache_rows(cache, b, L + n, block_table, page_size)[L:L + n]
+    return out
+
+
+def tree_attn(q: np.ndarray, tree_k: Optional[np.ndarray], tree_v: Optional[np.ndarray],
               k_cache: np.ndarray, v_cache: np.ndarray, cache_len: np.ndarray,
               n_nodes: np.ndarray, anc: np.ndarray, scale: float,
               block_table: Optional[np.ndarray] = None, page_size: int = 16,
@@ -265,9 +281,13 @@ def tree_attn(q: np.ndarray, tree_k: np.ndarray, tree_v: np.ndarray,
     Query node j of sequence b, head h (kv head h // G) attends to the cached
     keys 0..L_b-1 and to the tree keys of its ancestors (itself included),
     softmax(scale * q k^T) v, all in float64.  ``seqs`` restricts the work to
-    some sequences; other rows of the result stay zero.
+    some sequences; other rows of the result stay zero.  ``tree_k`` and
+    ``tree_v`` None: the in-place layout (node j's rows at cache slot L_b + j).
     """
     B, N, Hq, D = q.shape
+    if tree_k is None:
+        tree_k = tree_rows_in_cache(k_cache, cache_len, n_nodes, N, block_table, page_size)
+        tree_v = tree_rows_in_cache(v_cache, cache_len, n_nodes, N, block_table, page_size)
     Hkv = tree_k.shape[2]
     G = Hq // Hkv
     out = np.zeros((B, N, Hq, D), dtype=np.float64)
@@ -337,7 +357,7 @@ def accept(targ: np.ndarray, n_nodes: np.ndarray, tok: np.ndarray, parent: np.nd
 # --------------------------------------------------------------------------
 # S6: repair resynchronisation (Sec. 3.5, Alg. 1)
 # --------------------------------------------------------------------------
-def resync(k_caches: list, v_caches: list, tree_k: np.ndarray, tree_v: np.ndarray,
+def resync(k_caches: list, v_caches: list, tree_k: Optional[list], tree_v: Optional[list],
            path_nodes: np.ndarray, accept_len: np.ndarray, diverge: np.ndarray,
            out_tokens: np.ndarray, cache_len: np.ndarray, block: int,
            block_table: Optional[np.ndarray] = None, page_size: int = 16):
@@ -350,9 +370,23 @@ def resync(k_caches: list, v_caches: list, tree_k: np.ndarray, tree_v: np.ndarra
     tokens to replay into the draft are the path tokens from depth d to a and
     the target's next token (only that token on branch-0 wins).
     ``k_caches``/``v_caches`` are per-layer arrays, modified in place;
-    ``tree_k``/``tree_v`` are [layers][B][N][Hkv][D].
+    ``tree_k``/``tree_v`` are [layers][B][N][Hkv][D], or None for the in-place
+    layout, where the path rows are read from cache slots L_b + node (all of
+    them before any write).
     """
     B = len(cache_len)
+    if tree_k is None:
+        tree_k, tree_v = [], []
+        for l in range(len(k_caches)):
+            rk, rv = {}, {}
+            for b in range(B):
+                L = int(cache_len[b])
+                for t in range(int(accept_len[b]) + 1):
+                    node = int(path_nodes[b, t])
+                    rk[b, node] = cache_rows(k_caches[l], b, L + node + 1, block_table, page_size)[L + node].copy()
+                    rv[b, node] = cache_rows(v_caches[l], b, L + node + 1, block_table, page_size)[L + node].copy()
+            tree_k.append(rk)
+            tree_v.append(rv)
     new_len = np.array(cache_len, dtype=np.int64)
     draft_valid = np.zeros(B, dtype=np.int64)
     replay = np.full((B, block + 2), -1, dtype=np.int64)
@@ -364,13 +398,14 @@ def resync(k_caches: list, v_caches: list, tree_k: np.ndarray, tree_v: np.ndarra
             for t in range(a + 1):
                 node = int(path_nodes[b, t])
                 slot = L + t
+                kr, vr = tree_k[l][b, node], tree_v[l][b, node]
                 if block_table is None:
-                    k_caches[l][b, slot] = tree_k[l][b, node]
-                    v_caches[l][b, slot] = tree_v[l][b, node]
+                    k_caches[l][b, slot] = kr
+                    v_caches[l][b, slot] = vr
                 else:
                     page = int(block_table[b, slot // page_size])
-                    k_caches[l][page, slot % page_size] = tree_k[l][b, node]
-                    v_caches[l][page, slot % page_size] = tree_v[l][b, node]
+                    k_caches[l][page, slot % page_size] = kr
+                    v_caches[l][page, slot % page_size] = vr
         new_len[b] = L + a + 1
         d = int(diverge[b])
         if d >= 0:

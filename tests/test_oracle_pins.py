@@ -471,6 +471,61 @@ def test_tree_attn_equals_per_path_causal_sdpa(seed):
                 assert np.allclose(out[b, j, h], o, rtol=1e-11, atol=1e-12)
 
 
+def _in_place_caches(kc, vc, tk, tv, L, n, paged, ps=4):
+    """Caches holding each sequence's cache rows at slots 0..L_b-1 and its
+    tree rows at slots L_b + j (the in-place layout); paged through a
+    shuffled block table when asked."""
+    B, _, Hkv, D = kc.shape
+    cap = int(max(L[b] + n[b] for b in range(B)))
+    ck = np.zeros((B, cap, Hkv, D))
+    cv = np.zeros((B, cap, Hkv, D))
+    for b in range(B):
+        ck[b, :L[b]], cv[b, :L[b]] = kc[b, :L[b]], vc[b, :L[b]]
+        ck[b, L[b]:L[b] + n[b]], cv[b, L[b]:L[b] + n[b]] = tk[b, :n[b]], tv[b, :n[b]]
+    if not paged:
+        return ck, cv, None
+    per = (cap + ps - 1) // ps
+    table = np.random.default_rng(5).permutation(B * per).reshape(B, per)
+    pk = np.zeros((B * per, ps, Hkv, D))
+    pv = np.zeros((B * per, ps, Hkv, D))
+    for b in range(B):
+        for sl in range(cap):
+            pk[table[b, sl // ps], sl % ps] = ck[b, sl]
+            pv[table[b, sl // ps], sl % ps] = cv[b, sl]
+    return pk, pv, table
+
+
+@pytest.mark.parametrize("paged", [False, True])
+@pytest.mark.parametrize("seed", range(3))
+def test_tree_attn_in_place_equals_per_path_causal_sdpa(seed, paged):
+    """The in-place layout (tree rows at cache slots L_b + j): the same
+    attention as per-path causal SDPA over the explicit path."""
+    q, tk, tv, kc, vc, L, t, D = _attn_case(seed)
+    n = t["n_nodes"]
+    ck, cv, table = _in_place_caches(kc, vc, tk, tv, L, n, paged)
+    scale = 1.0 / math.sqrt(D)
+    out = oracle.tree_attn(q, None, None, ck, cv, L, n, t["anc"], scale, block_table=table, page_size=4)
+    B, N, Hq, _ = q.shape
+    G = Hq // tk.shape[2]
+    for b in range(B):
+        for j in range(int(n[b])):
+            path = []
+            x = j
+            while x >= 0:
+                path.append(x)
+                x = int(t["parent"][b, x])
+            path = path[::-1]
+            for h in range(Hq):
+                hk = h // G
+                ks = np.concatenate([kc[b, :L[b], hk], tk[b, path, hk]])
+                vs = np.concatenate([vc[b, :L[b], hk], tv[b, path, hk]])
+                Tq = torch.from_numpy(np.concatenate([np.zeros((len(ks) - 1, D)), q[b, j, h][None]]))
+                o = torch.nn.functional.scaled_dot_product_attention(
+                    Tq[None, None], torch.from_numpy(ks)[None, None], torch.from_numpy(vs)[None, None],
+                    is_causal=True, scale=scale)[0, 0, -1].numpy()
+                assert np.allclose(out[b, j, h], o, rtol=1e-11, atol=1e-12)
+
+
 def test_tree_attn_constant_keys_give_mean_of_values():
     q, tk, tv, kc, vc, L, t, D = _attn_case(11)
     kc[:] = 0.3
@@ -651,6 +706,33 @@ def test_resync_paged_matches_contiguous():
         for s in range(128):
             assert np.array_equal(cont_k[l][0, s], pag_k[l][table[0, s // ps], s % ps])
             assert np.array_equal(cont_v[l][0, s], pag_v[l][table[0, s // ps], s % ps])
+
+
+@pytest.mark.parametrize("case", ["repair_win", "branch0_win"])
+def test_resync_in_place_hand(case):
+    """In-place resync: the path rows come from cache slots L + node.  The
+    result at slots L..L+a is the path's rows by depth; rows of chain nodes
+    are already in place, so only the repair nodes' rows change slots."""
+    g, t, c, r = _hand_accept(case)
+    L, K = g["cache_len"], g["K"]
+    n = int(t["n_nodes"][0])
+    rng = np.random.default_rng(3)
+    Hkv, D = 2, 4
+    ck = [rng.standard_normal((1, L + n + 4, Hkv, D)) for _ in range(2)]
+    cv = [rng.standard_normal((1, L + n + 4, Hkv, D)) for _ in range(2)]
+    before_k = [x.copy() for x in ck]
+    oracle.resync(ck, cv, None, None, r["path_nodes"], r["accept_len"], r["diverge_depth"],
+                  r["out_tokens"], np.array([L]), K)
+    a = int(r["accept_len"][0])
+    path = [int(x) for x in r["path_nodes"][0, :a + 1]]
+    for l in range(2):
+        for d, node in enumerate(path):
+            assert np.array_equal(ck[l][0, L + d], before_k[l][0, L + node])
+        assert np.array_equal(ck[l][0, :L], before_k[l][0, :L])   # the old cache is untouched
+        moved = [d for d, node in enumerate(path) if node != d]
+        assert all(node > K for d, node in enumerate(path) if node != d)
+        if case == "branch0_win":
+            assert moved == [] and np.array_equal(ck[l], before_k[l])
 
 
 # ---------------------------------------------------------------- pin power
