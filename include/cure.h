@@ -159,7 +159,13 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
  *                  the tree keys a with bit a of anc[b][j] set.
  * q, out: bf16 [B][n_max][heads_q][D]; tree_k, tree_v: bf16 [B][n_max][heads_kv][D]
  * (this step's target keys/values of the tree tokens); k_cache, v_cache: one
- * layer in the layout of `kv` (a HOST pointer).  Accumulation is float32; the
+ * layer in the layout of `kv` (a HOST pointer).
+ * In-place layout: tree_k = tree_v = NULL means the tree rows were written
+ * into the cache itself, node j of sequence b at slot L_b + j (a paged cache
+ * then needs block_table entries up to slot L_b + n_b - 1).  The keys are then
+ * one range 0..L_b+n_b-1 of the cache, in 64-key tiles; a tile past L_b
+ * masks its tree part with the ancestor bits.  L_b + n_b past the capacity
+ * sets CURE_DEVERR_SLOT.  Accumulation is float32; the
  * probabilities are rounded to bf16 before the PV product.  D = 128,
  * heads_q % heads_kv == 0, scale > 0 and finite (1/sqrt(D) in the paper's
  * models; otherwise CURE_ERR_INVALID_ARG), all tensor base pointers 16-byte
@@ -238,6 +244,10 @@ cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch,
  * For every layer l and sequence b, the K/V rows of the accepted path's nodes
  * at depths 0..a are copied from tree_k/tree_v (bf16 [layers][B][n_max][Hkv][D])
  * into cache slots L_b..L_b+a of k_caches[l]/v_caches[l] (layout `kv`).
+ * In-place layout (tree_k = tree_v = NULL, see cure_tree_attn): node j's rows
+ * are read from cache slot L_b + j, so the rows of branch-0 nodes (j = depth)
+ * are already in place and only the repair nodes past the divergence depth
+ * are copied (nothing when branch 0 wins).
  * Then cache_len_out[b] = L_b + a + 1, draft_valid_len[b] = L_b + d when a
  * repair path wins at divergence depth d (else L_b + a + 1), and
  * replay_tokens[b] (int32 [B][K+2]) = the path tokens at depths d..a followed by

@@ -16,6 +16,7 @@ struct AttnArgs {
   const int32_t* n_nodes;
   const uint64_t* anc;
   int batch, n_max, heads_q, G, W, cap;
+  int inplace;     // 1: no tree tensors; node j's K/V rows are cache slot L_b + j
   int units_max;   // piece counters in the workspace
   int unit_cost;   // fixed cost of a unit in the stream-K split, in 64-key tile times
   float scale_log2;

@@ -154,7 +154,8 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
   if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
     return CURE_ERR_UNSUPPORTED;
   if (batch == 0) return CURE_OK;
-  if (!q || !tree_k || !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out ||
+  // tree_k and tree_v both NULL: the in-place layout (tree rows at cache slots L_b + j)
+  if (!q || !tree_k != !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out ||
       !workspace)
     return CURE_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(tree_k, 16) || !aligned(tree_v, 16) || !aligned(k_cache, 16) ||
@@ -217,7 +218,8 @@ cure_status cure_resync_kv(int32_t layers, void* const* k_caches, void* const* v
     return CURE_ERR_INVALID_ARG;
   LayerPtrs lp;
   if (layers > 0) {
-    if (!k_caches || !v_caches || !tree_k || !tree_v || !aligned(tree_k, 16) ||
+    // tree_k and tree_v both NULL: the in-place layout (tree rows at cache slots L_b + j)
+    if (!k_caches || !v_caches || !tree_k != !tree_v || !aligned(tree_k, 16) ||
         !aligned(tree_v, 16))
       return CURE_ERR_INVALID_ARG;
     for (int l = 0; l < layers; ++l) {

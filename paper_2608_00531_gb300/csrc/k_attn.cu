@@ -43,6 +43,7 @@ cudaError_t launch_tree_attn(const AttnPlan& plan, const uint16_t* q, const uint
   A.q = q;
   A.tk = tree_k;
   A.tv = tree_v;
+  A.inplace = tree_k == nullptr ? 1 : 0;
   A.kc = k_cache;
   A.vc = v_cache;
   A.kv = kv;

@@ -284,6 +284,7 @@ struct Sched {
   const int* cache_len;
   const int* n_nodes;
   int cap, n_max;
+  int inplace;             // tree rows at cache slots L + j: one key range [0, L + n)
   __device__ int owner(long long g) const {  // the CTA whose range holds position g
     return (int)(((g + 1) * (long long)P - 1) / Ttot);
   }
@@ -302,8 +303,11 @@ struct Sched {
     s.b = lo;
     s.L = max(0, min(cache_len[lo], cap));
     s.n = max(1, min(n_nodes[lo], n_max));
-    s.nct = (s.L + BN - 1) / BN;
-    s.T = s.nct + (s.n + BN - 1) / BN;
+    if (inplace && s.L + s.n > cap) s.L = max(0, cap - s.n);
+    // cache tiles (0..nct-1), then the tree tiles of separate tree tensors;
+    // in the in-place layout every tile is a cache tile over keys 0..L+n-1
+    s.nct = ((inplace ? s.L + s.n : s.L) + BN - 1) / BN;
+    s.T = inplace ? s.nct : s.nct + (s.n + BN - 1) / BN;
     const long long local = g - tiles_start[lo];
     const int Tc = s.T + C;
     const int uib = (int)(local / Tc);
@@ -399,9 +403,14 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_NODES);
           n = max(1, min(n, A.n_max));
         }
+        if (A.inplace && L + n > A.cap) {  // the tree rows must fit in the cache
+          if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_SLOT);
+          L = max(0, A.cap - n);
+        }
         const int rg = (n + 2 * npb - 1) / (2 * npb);
         ub = rg * Hkv;
-        tb = ub * ((L + BN - 1) / BN + (n + BN - 1) / BN + A.unit_cost);
+        const int T = A.inplace ? (L + n + BN - 1) / BN : (L + BN - 1) / BN + (n + BN - 1) / BN;
+        tb = ub * (T + A.unit_cost);
       }
       int it = tb, iu = ub;
 #pragma unroll
@@ -445,6 +454,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
   sch.n_nodes = A.n_nodes;
   sch.cap = A.cap;
   sch.n_max = A.n_max;
+  sch.inplace = A.inplace;
   const bool takes_part = (int)blockIdx.x < sch.P;
   const long long g_begin = takes_part ? (long long)blockIdx.x * sch.Ttot / sch.P : 0;
   const long long g_end = takes_part ? (long long)(blockIdx.x + 1) * sch.Ttot / sch.P : 0;
@@ -491,7 +501,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             pg[p] = -1;
             if (p < ppt && tl < s.nct && tl < s.t1) {
               const int tok = tl * BN + p * ps;
-              if (tok < s.L) {
+              if (tok < s.L + (A.inplace ? s.n : 0) && tok / ps < A.kv.max_len) {
                 const int page = A.kv.block_table[(int64_t)s.b * A.kv.max_len + tok / ps];
                 if (page < 0 || page >= A.kv.num_pages) flag(A.err, CURE_DEVERR_PAGE);
                 else pg[p] = page;  // a missing page stays -1: its box reads zeros
@@ -695,9 +705,36 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
 
           // raw scores, -inf where masked; the scale is applied in the exponent
           const bool tree = t >= s.nct;
-          const int valid = tree ? min(BN, s.n - (t - s.nct) * BN) : min(BN, s.L - t * BN);
+          const int kend = A.inplace ? s.L + s.n : s.L;  // keys of the cache tiles
+          const int valid = tree ? min(BN, s.n - (t - s.nct) * BN) : min(BN, kend - t * BN);
+          // in the in-place layout, a tile that reaches past L holds tree rows
+          // (key k is node k - L): cache keys below L are visible, tree keys
+          // through the row's ancestor bits, read at the tile's offset
+          const bool mixed = A.inplace && (t + 1) * BN > s.L;
           float x[64];
-          if (tree) {
+          if (mixed) {
+            const int off = t * BN - s.L;  // node of the tile's first key, > -64
+            uint64_t vis = 0ull;
+            if (vrow) {
+              const uint64_t* ar = A.anc + ((int64_t)s.b * A.n_max + node) * A.W;
+              if (off < 0) {
+                vis = (ar[0] << (-off)) | ((1ull << (-off)) - 1ull);
+              } else {
+                const int wi = off >> 6, sh = off & 63;
+                const uint64_t lo = wi < A.W ? ar[wi] : 0ull;
+                const uint64_t hi = (sh != 0 && wi + 1 < A.W) ? ar[wi + 1] : 0ull;
+                vis = (lo >> sh) | (sh != 0 ? hi << (64 - sh) : 0ull);
+              }
+            } else if (off < 0) {
+              vis = (1ull << (-off)) - 1ull;
+            }
+            const uint32_t w0 = (uint32_t)vis, w1 = (uint32_t)(vis >> 32);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              x[i] = ((w0 >> i) & 1u) ? __uint_as_float(u0[i]) : -INFINITY;
+              x[32 + i] = ((w1 >> i) & 1u) ? __uint_as_float(u1[i]) : -INFINITY;
+            }
+          } else if (tree) {
             const int wi = t - s.nct;
             const uint64_t word = vrow ? A.anc[((int64_t)s.b * A.n_max + node) * A.W + wi] : 0ull;
             const uint32_t w0 = (uint32_t)word, w1 = (uint32_t)(word >> 32);
@@ -1061,7 +1098,11 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
          make_page_map(&mv, A.vc, (uint64_t)A.kv.num_pages, ps, Hkv);
   }
   const uint64_t trows = (uint64_t)A.batch * A.n_max;
-  ok = ok && make_kv_map(&mtk, A.tk, trows, Hkv, BN) && make_v_rows_map(&mtv, A.tv, trows, Hkv) &&
+  // in the in-place layout the tree maps are never used for a copy; they are
+  // encoded over Q (at least as large) so that every map passed is valid
+  const void* tk = A.inplace ? static_cast<const void*>(A.q) : A.tk;
+  const void* tv = A.inplace ? static_cast<const void*>(A.q) : A.tv;
+  ok = ok && make_kv_map(&mtk, tk, trows, Hkv, BN) && make_v_rows_map(&mtv, tv, trows, Hkv) &&
        make_q_map(&mq, A.q, trows, Hkv, A.G, BM / A.G);
   if (!ok) return cudaErrorInvalidValue;
   // a fresh tag per launch makes the piece counters left in the workspace

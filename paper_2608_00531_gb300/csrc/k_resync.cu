@@ -1,7 +1,10 @@
 // Stage 6: repair resynchronisation (Sec. 3.5, Alg. 1 last step).
 //
 // gather: one warp per (sequence, depth, K|V, group of kLayersPerWarp layers);
-// warps past the accepted length leave at once.  The warp resolves the
+// warps past the accepted length leave at once.  With no tree tensors (the
+// in-place layout, node j's rows at cache slot L + j) the path rows come from
+// the cache itself, and a branch-0 node, whose slot L + j is already its
+// depth's, copies nothing: only the rows past the divergence move.  The warp resolves the
 // path row once (tree node, cache row through the block table) and copies
 // the row of each layer of its group: heads_kv * head_dim bf16 values
 // (1 KiB for 4 x 128) as 16-byte vectors, all the group's loads in flight
@@ -73,28 +76,35 @@ resync_gather_kernel(int layers, LayerPtrs caches, cure_kv_desc kv, const uint4*
     if (lane == 0) flag(err, CURE_DEVERR_NODES);
     return;
   }
-  const int slot = cache_len_in[b] + t;
+  const bool inplace = tree_k == nullptr;
+  if (inplace && node == t) return;  // already in its slot
   const int row_vec = kv.heads_kv * kv.head_dim / 8;  // uint4 per row
-  int64_t dst_row;
-  if (kv.layout == 0) {
-    if (slot < 0 || slot >= kv.max_len) {
-      if (lane == 0) flag(err, CURE_DEVERR_SLOT);
-      return;
+  // the cache row of slot `slot`, or -1 (error word set) when it does not exist
+  auto row_of = [&](int slot) -> int64_t {
+    if (kv.layout == 0) {
+      if (slot < 0 || slot >= kv.max_len) {
+        if (lane == 0) flag(err, CURE_DEVERR_SLOT);
+        return -1;
+      }
+      return (int64_t)b * kv.max_len + slot;
     }
-    dst_row = (int64_t)b * kv.max_len + slot;
-  } else {
     const int pi = slot / kv.page_size;
     if (slot < 0 || pi >= kv.max_len) {
       if (lane == 0) flag(err, CURE_DEVERR_SLOT);
-      return;
+      return -1;
     }
     const int page = kv.block_table[(int64_t)b * kv.max_len + pi];
     if (page < 0 || page >= kv.num_pages) {
       if (lane == 0) flag(err, CURE_DEVERR_PAGE);
-      return;
+      return -1;
     }
-    dst_row = (int64_t)page * kv.page_size + slot % kv.page_size;
-  }
+    return (int64_t)page * kv.page_size + slot % kv.page_size;
+  };
+  const int L = cache_len_in[b];
+  const int64_t dst_row = row_of(L + t);
+  if (dst_row < 0) return;
+  const int64_t src_row = inplace ? row_of(L + node) : 0;
+  if (src_row < 0) return;
   const uint4* tree = which == 0 ? tree_k : tree_v;
   const int l0 = group * kLayersPerWarp, nl = min(kLayersPerWarp, layers - l0);
   for (int i0 = lane; i0 < row_vec; i0 += 32 * 2) {  // two vectors per lane per layer
@@ -102,7 +112,10 @@ resync_gather_kernel(int layers, LayerPtrs caches, cure_kv_desc kv, const uint4*
 #pragma unroll
     for (int q = 0; q < kLayersPerWarp; ++q) {
       if (q < nl) {
-        const uint4* src = tree + ((((int64_t)(l0 + q) * batch + b) * n_max + node) * row_vec);
+        const uint4* src =
+            inplace ? reinterpret_cast<const uint4*>(which == 0 ? caches.k[l0 + q] : caches.v[l0 + q]) +
+                          src_row * row_vec
+                    : tree + ((((int64_t)(l0 + q) * batch + b) * n_max + node) * row_vec);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
           if (i0 + 32 * h < row_vec) v[q][h] = __ldg(src + i0 + 32 * h);

@@ -122,15 +122,19 @@ def cure_tree_attn_workspace_size(batch: int, n_max: int, heads_q: int, kv: KVDe
     return int(_lib.load().cure_tree_attn_workspace_size(batch, n_max, heads_q, C.byref(kv)))
 
 
-def cure_tree_attn(q: torch.Tensor, tree_k: torch.Tensor, tree_v: torch.Tensor,
+def cure_tree_attn(q: torch.Tensor, tree_k: Optional[torch.Tensor], tree_v: Optional[torch.Tensor],
                    k_cache: torch.Tensor, v_cache: torch.Tensor, kv: KVDesc,
                    cache_len: torch.Tensor, n_nodes: torch.Tensor, anc: torch.Tensor,
                    scale: float, *, out: Optional[torch.Tensor] = None,
                    workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    """Stage 4 (Sec. 3.2/3.4/3.5): tree-masked GQA attention for one layer."""
+    """Stage 4 (Sec. 3.2/3.4/3.5): tree-masked GQA attention for one layer.
+
+    tree_k = tree_v = None: the in-place layout, node j's K/V rows at cache
+    slot cache_len[b] + j."""
     for t, nm in ((q, "q"), (tree_k, "tree_k"), (tree_v, "tree_v"), (k_cache, "k_cache"),
                   (v_cache, "v_cache")):
-        _need(t, torch.bfloat16, nm)
+        if t is not None or nm not in ("tree_k", "tree_v"):
+            _need(t, torch.bfloat16, nm)
     B, n_max, Hq, D = q.shape
     if out is None:
         out = torch.empty_like(q)
@@ -180,16 +184,21 @@ def cure_accept(tree: dict, block: int, *, target_logits: Optional[torch.Tensor]
 
 
 def cure_resync_kv(k_caches: Sequence[torch.Tensor], v_caches: Sequence[torch.Tensor], kv: KVDesc,
-                   tree_k: torch.Tensor, tree_v: torch.Tensor, acc: dict,
-                   cache_len_in: torch.Tensor, block: int, *,
+                   tree_k: Optional[torch.Tensor], tree_v: Optional[torch.Tensor], acc: dict,
+                   cache_len_in: torch.Tensor, block: int, *, n_max: Optional[int] = None,
                    cache_len_out: Optional[torch.Tensor] = None, out=None, stream=None) -> dict:
     """Stage 6 (Sec. 3.5, Alg. 1): write the path into every layer's cache, realign the draft.
 
-    tree_k/tree_v: bf16 [layers][B][n_max][Hkv][D].
+    tree_k/tree_v: bf16 [layers][B][n_max][Hkv][D], or None for the in-place
+    layout (the path rows are then read from cache slots L + node, and only
+    the rows past the divergence move; give n_max).
     """
     layers = len(k_caches)
     B = cache_len_in.shape[0]
-    n_max = tree_k.shape[2] if layers else block + 1
+    if n_max is None:
+        if layers and tree_k is None:
+            raise ValueError("cure_resync_kv: the in-place layout needs n_max")
+        n_max = tree_k.shape[2] if layers else block + 1
     dev = cache_len_in.device
     P = block + 2
     if cache_len_out is None:

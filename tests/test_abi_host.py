@@ -89,6 +89,10 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
     assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 5
     kv.head_dim = 128
     assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 6, 1.0, null, null, 0, null) == 1
+    # the in-place layout passes both tree tensors as NULL, never only one of them
+    dev = C.c_void_p(256)
+    one = (dev, dev, null, dev, dev)
+    assert lib.cure_tree_attn(*one, C.byref(kv), dev, dev, dev, 1, 9, 8, 1.0, dev, dev, 1 << 30, null) == 1
     # the softmax scale must be positive and finite
     for bad in (0.0, -1.0, float("inf"), float("nan")):
         assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, bad, null, null, 0,

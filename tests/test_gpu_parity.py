@@ -384,6 +384,73 @@ def test_tree_attn_wide_tree_two_words(cure):
     _cmp_attn(got, ref, t)
 
 
+def _in_place_case(B, K, budget, Hq, Hkv, lens, paged, seed, tau=1.0, ps=16):
+    """An attention case in the in-place layout: caches with room for the
+    tree, node j's K/V rows written at cache slot L_b + j."""
+    t, q, tk, tv, _, _, L, _, _ = _attn_case(B, K, budget, Hq, Hkv, lens, False, 1.0, 1.0, seed, tau=tau)
+    rng = np.random.default_rng(seed + 1000)
+    N = 1 + K + budget
+    D = 128
+    if paged:
+        table, npages = W.block_table(L, N - 1, seed, ps)     # pages for slots 0..L_b + N - 1
+        kc = W.normal_bf16((npages, ps, Hkv, D), 1.0, rng)
+        vc = W.normal_bf16((npages, ps, Hkv, D), 1.0, rng)
+    else:
+        table, npages = None, 0
+        kc = W.normal_bf16((B, int(L.max()) + N + 3, Hkv, D), 1.0, rng)
+        vc = W.normal_bf16((B, int(L.max()) + N + 3, Hkv, D), 1.0, rng)
+    for b in range(B):
+        for j in range(int(t["n_nodes"][b])):
+            sl = int(L[b]) + j
+            if paged:
+                kc[table[b, sl // ps], sl % ps] = tk[b, j]
+                vc[table[b, sl // ps], sl % ps] = tv[b, j]
+            else:
+                kc[b, sl] = tk[b, j]
+                vc[b, sl] = tv[b, j]
+    return t, q, kc, vc, L, table, npages
+
+
+def _run_attn_in_place(c, t, q, kc, vc, L, table, npages, Hkv):
+    if table is not None:
+        kv = c.kv_desc(Hkv, 128, table.shape[1], torch.from_numpy(table).to(DEV), kc.shape[1], npages)
+    else:
+        kv = c.kv_desc(Hkv, 128, kc.shape[1])
+    out = c.cure_tree_attn(q.to(DEV), None, None, kc.to(DEV), vc.to(DEV), kv, torch.from_numpy(L).to(DEV),
+                           torch.from_numpy(t["n_nodes"].astype(np.int32)).to(DEV),
+                           torch.from_numpy(t["anc"].view(np.int64)).to(DEV), 1.0 / math.sqrt(128))
+    torch.cuda.synchronize()
+    assert c.cure_device_error() == 0
+    return out.float().cpu().numpy()
+
+
+@pytest.mark.parametrize("paged", [False, True])
+@pytest.mark.parametrize("Hq,Hkv", [(8, 2), (28, 4), (32, 8)])
+def test_tree_attn_in_place(cure, paged, Hq, Hkv):
+    """The in-place layout: cache lengths that put the tree at every kind of
+    tile offset (L = 0, inside the first tile, L a multiple of 64, one key
+    before a tile boundary, several tiles, more than one split)."""
+    lens = [0, 37, 64, 127, 700, 2100]
+    t, q, kc, vc, L, table, npages = _in_place_case(6, 8, 6, Hq, Hkv, lens, paged, seed=40 + Hq)
+    got = _run_attn_in_place(cure, t, q, kc, vc, L, table, npages, Hkv)
+    ref = oracle.tree_attn(_f64(q), None, None, _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128), table, 16)
+    _cmp_attn(got, ref, t)
+
+
+@pytest.mark.parametrize("paged", [False, True])
+def test_tree_attn_in_place_two_words(cure, paged):
+    """97-node trees in the in-place layout: the ancestor window of a tile
+    straddles the two words at every bit offset."""
+    lens = [300, 1500, 1, 63, 64, 65]
+    t, q, kc, vc, L, table, npages = _in_place_case(6, 32, 64, 28, 4, lens, paged, seed=8, tau=4.0)
+    assert t["n_nodes"].max() > 64
+    got = _run_attn_in_place(cure, t, q, kc, vc, L, table, npages, 4)
+    ref = oracle.tree_attn(_f64(q), None, None, _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128), table, 16)
+    _cmp_attn(got, ref, t)
+
+
 def test_tree_attn_full_serve_layer_sampled(cure):
     """One layer at the benchmark's serving shape (batch 32, 28/4 heads, paged
     16-token blocks, lengths U[1024, 8192]); the oracle checks 3 sequences."""
@@ -538,6 +605,48 @@ def test_resync(cure, paged):
     ko = [_f64(x) for x in kcs]
     vo = [_f64(x) for x in vcs]
     o_rs = oracle.resync(ko, vo, _f64(tk), _f64(tv), o_acc["path_nodes"], o_acc["accept_len"],
+                         o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, paged or 16)
+    for key in ("cache_len", "draft_valid_len", "replay_tokens", "n_replay"):
+        assert np.array_equal(rs[key].cpu().numpy(), o_rs[key]), key
+    for l in range(layers):
+        assert np.array_equal(_f64(kd[l].cpu()), ko[l])
+        assert np.array_equal(_f64(vd[l].cpu()), vo[l])
+
+
+@pytest.mark.parametrize("paged", [0, 16])
+def test_resync_in_place_layout(cure, paged):
+    """The in-place layout: the path rows come from cache slots L + node and
+    only the repair rows move; the whole cache must match the oracle."""
+    rng = np.random.default_rng(31 + int(paged))
+    B, K, budget, Hkv, D, layers = 6, 8, 6, 4, 128, 3
+    margin = (rng.integers(0, 8, size=(B, K)) * 0.25).astype(np.float32)
+    ids = np.tile(np.arange(3), (B, K, 1))
+    t = oracle.build_tree(ids, margin, rng.integers(0, 3, size=B), rng.integers(0, 99, size=B), 1.5,
+                          budget, 3, 1)
+    targ = rng.integers(0, 3, size=t["tok"].shape)
+    o_acc = oracle.accept(targ, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], K)
+    assert (o_acc["diverge_depth"] >= 0).any() and (o_acc["diverge_depth"] < 0).any()
+    L = rng.integers(0, 200, size=B).astype(np.int32)
+    N = 1 + K + budget
+    if paged:
+        table, npages = W.block_table(L, N - 1, 5, paged)
+        shape = (npages, paged, Hkv, D)
+        kv = cure.kv_desc(Hkv, D, table.shape[1], torch.from_numpy(table).to(DEV), paged, npages)
+    else:
+        table = None
+        shape = (B, int(L.max()) + N + 1, Hkv, D)
+        kv = cure.kv_desc(Hkv, D, shape[1])
+    kcs = [W.normal_bf16(shape, 1.0, rng) for _ in range(layers)]
+    vcs = [W.normal_bf16(shape, 1.0, rng) for _ in range(layers)]
+    kd = [x.to(DEV) for x in kcs]
+    vd = [x.to(DEV) for x in vcs]
+    acc = {k_: torch.from_numpy(v.astype(np.int32)).to(DEV) for k_, v in o_acc.items()}
+    rs = cure.cure_resync_kv(kd, vd, kv, None, None, acc, torch.from_numpy(L).to(DEV), K, n_max=N)
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    ko = [_f64(x) for x in kcs]
+    vo = [_f64(x) for x in vcs]
+    o_rs = oracle.resync(ko, vo, None, None, o_acc["path_nodes"], o_acc["accept_len"],
                          o_acc["diverge_depth"], o_acc["out_tokens"], L, K, table, paged or 16)
     for key in ("cache_len", "draft_valid_len", "replay_tokens", "n_replay"):
         assert np.array_equal(rs[key].cpu().numpy(), o_rs[key]), key
