@@ -35,7 +35,7 @@ import torch  # noqa: E402
 # DRAM bytes (read + write) of one tree-attention launch on this workload, from
 # one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
 # source with the given sha256 prefix; another source reports null
-ATTN_TRAFFIC = {"c0b2103f24736b70": 313095424}
+ATTN_TRAFFIC = {"2d1748d0f70bce81": 312700160}
 
 METRIC = "repair-verify steps/s at batch 32, block 16; tree-attn & vocab-scan HBM GB/s vs peak"
 WORKLOAD = "serve32"

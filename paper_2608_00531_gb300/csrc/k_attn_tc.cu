@@ -284,7 +284,7 @@ struct Sched {
   const int* cache_len;
   const int* n_nodes;
   int cap, n_max;
-  int inplace;             // tree rows at cache slots L + j: one key range [0, L + n)
+  bool inplace;            // tree rows at cache slots L + j: one key range [0, L + n)
   __device__ int owner(long long g) const {  // the CTA whose range holds position g
     return (int)(((g + 1) * (long long)P - 1) / Ttot);
   }
@@ -328,6 +328,10 @@ struct Sched {
   }
 };
 
+// INPLACE: the in-place layout (no tree tensors; node j's rows at cache slot
+// L + j), a template parameter so that the separate-tensor kernel carries
+// none of its tests.
+template <bool INPLACE>
 __global__ void __launch_bounds__(kThreads, 1)
 tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                     const __grid_constant__ CUtensorMap tm_tk, const __grid_constant__ CUtensorMap tm_tv,
@@ -403,13 +407,13 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_NODES);
           n = max(1, min(n, A.n_max));
         }
-        if (A.inplace && L + n > A.cap) {  // the tree rows must fit in the cache
+        if (INPLACE && L + n > A.cap) {  // the tree rows must fit in the cache
           if (blockIdx.x == 0) flag(A.err, CURE_DEVERR_SLOT);
           L = max(0, A.cap - n);
         }
         const int rg = (n + 2 * npb - 1) / (2 * npb);
         ub = rg * Hkv;
-        const int T = A.inplace ? (L + n + BN - 1) / BN : (L + BN - 1) / BN + (n + BN - 1) / BN;
+        const int T = INPLACE ? (L + n + BN - 1) / BN : (L + BN - 1) / BN + (n + BN - 1) / BN;
         tb = ub * (T + A.unit_cost);
       }
       int it = tb, iu = ub;
@@ -454,7 +458,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
   sch.n_nodes = A.n_nodes;
   sch.cap = A.cap;
   sch.n_max = A.n_max;
-  sch.inplace = A.inplace;
+  sch.inplace = INPLACE;
   const bool takes_part = (int)blockIdx.x < sch.P;
   const long long g_begin = takes_part ? (long long)blockIdx.x * sch.Ttot / sch.P : 0;
   const long long g_end = takes_part ? (long long)(blockIdx.x + 1) * sch.Ttot / sch.P : 0;
@@ -501,7 +505,7 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             pg[p] = -1;
             if (p < ppt && tl < s.nct && tl < s.t1) {
               const int tok = tl * BN + p * ps;
-              if (tok < s.L + (A.inplace ? s.n : 0) && tok / ps < A.kv.max_len) {
+              if (tok < s.L + (INPLACE ? s.n : 0) && tok / ps < A.kv.max_len) {
                 const int page = A.kv.block_table[(int64_t)s.b * A.kv.max_len + tok / ps];
                 if (page < 0 || page >= A.kv.num_pages) flag(A.err, CURE_DEVERR_PAGE);
                 else pg[p] = page;  // a missing page stays -1: its box reads zeros
@@ -705,12 +709,12 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
 
           // raw scores, -inf where masked; the scale is applied in the exponent
           const bool tree = t >= s.nct;
-          const int kend = A.inplace ? s.L + s.n : s.L;  // keys of the cache tiles
+          const int kend = INPLACE ? s.L + s.n : s.L;  // keys of the cache tiles
           const int valid = tree ? min(BN, s.n - (t - s.nct) * BN) : min(BN, kend - t * BN);
           // in the in-place layout, a tile that reaches past L holds tree rows
           // (key k is node k - L): cache keys below L are visible, tree keys
           // through the row's ancestor bits, read at the tile's offset
-          const bool mixed = A.inplace && (t + 1) * BN > s.L;
+          const bool mixed = INPLACE && (t + 1) * BN > s.L;
           float x[64];
           if (mixed) {
             const int off = t * BN - s.L;  // node of the tile's first key, > -64
@@ -1081,8 +1085,11 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if (!(attr_done.load() & bit)) {
-    e = cudaFuncSetAttribute(tree_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(tree_attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(tree_attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_done.fetch_or(bit);
   }
@@ -1110,7 +1117,10 @@ cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s) {
   static std::atomic<uint32_t> launches{0};
   AttnArgs a = A;
   a.tag = launches.fetch_add(1) % ((1u << (32 - kCountBits)) - 1) + 1;
-  e = launch_pdl(tree_attn_tc_kernel, grid, dim3(kThreads), kSmemBytes, s, mk, mv, mtk, mtv, mq, a);
+  e = A.inplace ? launch_pdl(tree_attn_tc_kernel<true>, grid, dim3(kThreads), kSmemBytes, s, mk, mv, mtk,
+                             mtv, mq, a)
+                : launch_pdl(tree_attn_tc_kernel<false>, grid, dim3(kThreads), kSmemBytes, s, mk, mv, mtk,
+                             mtv, mq, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
