@@ -177,7 +177,8 @@ def make_workload(dev, rank: int, layers_override=None, pool: int = POOL):
     layers = layers_override or w.layers
     B, K, N, D = w.batch, w.block, w.n_max, 128
     L = W.cache_lengths(w, seed=seed)
-    table, npages = W.block_table(L, K, seed)
+    # pages for slots up to L_b + n_max - 1: room for the in-place layout's tree rows
+    table, npages = W.block_table(L, N - 1, seed)
     g = torch.Generator(device=dev).manual_seed(seed)
 
     def rnd(*shape, std=1.0):
@@ -437,6 +438,12 @@ def main():
     if not args.no_e2e:
         e2e = run_e2e(wl, st, kcs, vcs, dev, max(3, min(args.steps, 10)), world)
 
+    # the in-place tree-KV layout on the same shapes; last, since its resync
+    # moves rows inside the caches
+    in_place = None
+    if not args.no_graph:
+        in_place = in_place_stage(st, xs[sel[-1]], kcs, vcs)
+
     if rank != 0:
         return
     pk = peaks()
@@ -488,7 +495,7 @@ def main():
                    "tree_attn_tflops": round(attn_tflops, 1), "tree_attn_intensity_flop_per_byte": round(intensity, 1),
                    "mean_tree_nodes": round(alg["mean_nodes"], 3),
                    "mean_accept_len": round(float(np.mean([acc_lens[i].mean() for i in sel])), 3),
-                   "input_sets": P},
+                   "input_sets": P, "in_place": in_place},
         "gpu_launches": st.launches_per_step * args.steps,
         "clocks": clocks,
     }
@@ -499,6 +506,40 @@ def main():
     if not args.no_cpu_baseline and world == 1:
         out["cpu_baseline"] = cpu_baseline()
     print(json.dumps(out), flush=True)
+
+
+def in_place_stage(st, x, kcs, vcs):
+    """The in-place tree-KV layout (node j's K/V rows at cache slot L + j, no
+    tree tensors) on the step's shapes: the layers of tree attention replayed
+    as a CUDA graph, per layer, and the resync call, replayed alone.  The cache
+    contents are the bench's random rows: these are timings, not results."""
+    try:
+        from paper_2608_00531_gb300 import cure
+        tree, Ly = st.tree, st.layers
+
+        def attn():
+            for l in range(Ly):
+                p = st.layer_map[l]
+                cure.cure_tree_attn(x.q[l], None, None, kcs[p], vcs[p], st.kv, x.cache_len, tree["n_nodes"],
+                                    tree["anc"], st.scale, out=st.attn_out[l], workspace=st.workspace)
+
+        def resync():
+            kl = [kcs[st.layer_map[l]] for l in range(Ly)]
+            vl = [vcs[st.layer_map[l]] for l in range(Ly)]
+            cure.cure_resync_kv(kl, vl, st.kv, None, None, st.acc, x.cache_len, st.K, n_max=st.n_max,
+                                cache_len_out=st.cache_len_out, out=st.rs)
+
+        a_ms = call_graph_ms(attn, calls=2, reps=5)
+        r_ms = call_graph_ms(resync)
+        if cure.cure_device_error() != 0:
+            return None
+        return {"tree_attn_ms_per_layer": None if a_ms is None else round(a_ms / Ly, 4),
+                "resync_graph_ms": None if r_ms is None else round(r_ms, 4),
+                "note": "tree rows written by the target at cache slots L + j; resync moves only the rows "
+                        "past the divergence depth"}
+    except Exception as e:  # reported as missing, the bench line stands
+        print(f"in-place timing failed: {type(e).__name__}: {e}"[:300], file=sys.stderr)
+        return None
 
 
 def call_graph_ms(fn, calls=20, reps=5):
