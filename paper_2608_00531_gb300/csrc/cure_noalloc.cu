@@ -72,7 +72,8 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
   if (n_max > kMaxNodes || batch > kAttnBatchLimit || heads_q / kv->heads_kv > 128)
     return CURE_ERR_UNSUPPORTED;
   if (batch == 0) return CURE_OK;
-  if (!q || !tree_k || !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out)
+  // tree_k and tree_v both NULL: the in-place layout, as in cure_tree_attn
+  if (!q || !tree_k != !tree_v || !k_cache || !v_cache || !cache_len || !n_nodes || !anc || !out)
     return CURE_ERR_INVALID_ARG;
   const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(tree_k) |
                         reinterpret_cast<uintptr_t>(tree_v) | reinterpret_cast<uintptr_t>(k_cache) |

@@ -63,10 +63,11 @@ def _inputs(seed, B=4, K=16, budget=16, Hq=28, Hkv=4, lens=(0, 37, 1500, 4000)):
                 anc=torch.from_numpy(t["anc"].view(np.int64)).to(DEV))
 
 
-def _call_noalloc(lib, x, kv, out):
+def _call_noalloc(lib, x, kv, out, in_place=False):
     s = C.c_void_p(torch.cuda.current_stream().cuda_stream)
+    tk, tv = (None, None) if in_place else (x["tk"].data_ptr(), x["tv"].data_ptr())
     return lib.cure_tree_attn_noalloc(
-        x["q"].data_ptr(), x["tk"].data_ptr(), x["tv"].data_ptr(), x["kc"].data_ptr(), x["vc"].data_ptr(),
+        x["q"].data_ptr(), tk, tv, x["kc"].data_ptr(), x["vc"].data_ptr(),
         C.byref(kv), x["L"].data_ptr(), x["n"].data_ptr(), x["anc"].data_ptr(), x["B"], x["N"], x["Hq"],
         1.0 / math.sqrt(128), out.data_ptr(), s)
 
@@ -89,6 +90,38 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(env):
             want = ref[b, :nb].float()
             assert torch.isfinite(got).all(), (call, b)
             assert float((got - want).abs().max()) <= TOL, (call, b)
+
+
+def test_noalloc_in_place_layout(env):
+    """Both tree tensors NULL: the in-place layout (node j's rows at cache
+    slot L + j), as in cure_tree_attn."""
+    lib, cure = env
+    x = _inputs(4)
+    L = x["L"].cpu().numpy()
+    table, npages = W.block_table(L, x["N"] - 1, 4)      # pages up to slot L + N - 1
+    rng = np.random.default_rng(4)
+    kc = W.normal_bf16((npages, 16, x["Hkv"], 128), 1.0, rng).to(DEV)
+    vc = W.normal_bf16((npages, 16, x["Hkv"], 128), 1.0, rng).to(DEV)
+    for b in range(x["B"]):
+        for j in range(int(x["t"]["n_nodes"][b])):
+            sl = int(L[b]) + j
+            kc[int(table[b, sl // 16]), sl % 16] = x["tk"][b, j]
+            vc[int(table[b, sl // 16]), sl % 16] = x["tv"][b, j]
+    x = dict(x, kc=kc, vc=vc, table=torch.from_numpy(table).to(DEV), npages=npages)
+    kv = cure.kv_desc(x["Hkv"], 128, table.shape[1], x["table"], 16, npages)
+    ref = cure.cure_tree_attn(x["q"], None, None, kc, vc, kv, x["L"], x["n"], x["anc"], 1.0 / math.sqrt(128))
+    sep = cure.cure_tree_attn(x["q"], x["tk"], x["tv"], kc, vc, kv, x["L"], x["n"], x["anc"],
+                              1.0 / math.sqrt(128))
+    out = torch.full_like(ref, float("nan"))
+    assert _call_noalloc(lib, x, kv, out, in_place=True) == 0
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+    for b in range(x["B"]):
+        nb = int(x["t"]["n_nodes"][b])
+        got = out[b, :nb].float()
+        assert torch.isfinite(got).all(), b
+        assert float((got - ref[b, :nb].float()).abs().max()) <= TOL, b
+        assert float((got - sep[b, :nb].float()).abs().max()) <= TOL, b     # the same attention
 
 
 def test_noalloc_rejects_shapes_beyond_its_scratch(env):
