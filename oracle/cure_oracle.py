@@ -15,6 +15,9 @@ Stages and the passages they follow:
                    construction, branch 0 anchored)
 * ``tree_attn``    Sec. 3.2 / 3.4 / 3.5 (single-pass Tree Attention)
 * ``accept``       Sec. 3.5 Eq. (4) with greedy decoding (Sec. 4.1)
+* ``sample_target`` the target's token per node at a temperature T > 0
+                   (Sec. 2: lossless speculative sampling; the paper's own
+                   runs are greedy, Sec. 4.1)
 * ``resync``       Sec. 3.5 and Alg. 1 (cache resynchronisation)
 
 Readings where the paper is silent or ambiguous (each is listed in the design
@@ -39,6 +42,12 @@ notes of the repository):
   costs one node, as at the last position); with a beam width, an
   alternative is admitted only if every depth it occupies still holds fewer
   nodes than the beam, the chain node included;
+* stochastic verification (T > 0) draws the target's token at every tree
+  node from softmax(logits / T) by inverse CDF with a given uniform u in
+  [0, 1): the first id whose cumulative probability exceeds u; the walk then
+  matches children against these samples as it matches them against the
+  argmax when greedy.  A sample is independent of the drafted children, so
+  every emitted token follows the target's distribution (lossless);
 * the best path is the deepest accepted node, lowest node index on ties;
 * resync writes the path's rows (root included) into cache slots L..L+a and
   realigns the draft to L + divergence depth (or L + a + 1 on branch-0 wins);
@@ -352,6 +361,34 @@ def accept(targ: np.ndarray, n_nodes: np.ndarray, tok: np.ndarray, parent: np.nd
                 break
     return dict(accept_len=accept_len, best_node=best_node, path_nodes=path_nodes,
                 out_tokens=out_tokens, diverge_depth=diverge)
+
+
+def sample_target(logits: np.ndarray, n_nodes: np.ndarray, uniforms: np.ndarray,
+                  temperature: float) -> np.ndarray:
+    """The target's token at each tree node, sampled at temperature T > 0.
+
+    Sec. 2 frames speculative decoding as lossless sampling from the target;
+    with T > 0 the target's token after node j is drawn from
+    softmax(logits[b][j] / T), here by inverse CDF: with u = uniforms[b][j] in
+    [0, 1), the first id v whose cumulative probability exceeds u.  A row of
+    -inf logits gives id 0 (as the argmax's tie rule would).  Rows at
+    j >= n_nodes[b] are -1.  Float64 throughout.
+    """
+    B, N, V = logits.shape
+    out = np.full((B, N), -1, dtype=np.int64)
+    for b in range(B):
+        for j in range(int(n_nodes[b])):
+            x = np.asarray(logits[b, j], dtype=np.float64)
+            m = x.max()
+            if m == -np.inf:
+                out[b, j] = 0
+                continue
+            p = np.exp((x - m) / temperature)
+            c = np.cumsum(p)
+            r = float(uniforms[b, j]) * c[-1]
+            y = int(np.searchsorted(c, r, side="right"))
+            out[b, j] = min(y, int(np.flatnonzero(p > 0)[-1]))
+    return out
 
 
 # --------------------------------------------------------------------------

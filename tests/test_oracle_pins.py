@@ -735,6 +735,48 @@ def test_resync_in_place_hand(case):
             assert moved == [] and np.array_equal(ck[l], before_k[l])
 
 
+# ------------------------------------------- stochastic verification pins
+def test_sample_target_closed_forms():
+    """Inverse-CDF sampling by hand: equal logits give floor(u V); two finite
+    logits a, b give the first id while u < e^(a/T) / (e^(a/T) + e^(b/T))."""
+    V = 10
+    x = np.zeros((1, 1, V))
+    for u in (0.0, 0.05, 0.31, 0.5, 0.99):
+        y = oracle.sample_target(x, np.array([1]), np.array([[u]]), 1.0)[0, 0]
+        assert y == math.floor(u * V), (u, y)
+    x = np.full((1, 1, V), -np.inf)
+    x[0, 0, 3], x[0, 0, 7] = 1.0, 2.0
+    for T in (0.5, 1.0, 3.0):
+        p3 = math.exp(1.0 / T) / (math.exp(1.0 / T) + math.exp(2.0 / T))
+        for u in (0.0, p3 - 1e-9, p3 + 1e-9, 0.999):
+            y = oracle.sample_target(x, np.array([1]), np.array([[u]]), T)[0, 0]
+            assert y == (3 if u < p3 else 7), (T, u, y)
+    # one finite logit: always that id; only -inf: id 0; rows past n_nodes: -1
+    x = np.full((1, 3, V), -np.inf)
+    x[0, 0, 6] = -4.0
+    y = oracle.sample_target(x, np.array([2]), np.array([[0.7, 0.2, 0.5]]), 1.0)
+    assert y[0].tolist() == [6, 0, -1]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_sample_target_frequencies_follow_softmax(seed):
+    """Over a fine grid of u, each id is drawn a share of the grid equal to
+    its softmax probability at T (to one grid step), and the draw never
+    decreases as u grows."""
+    rng = np.random.default_rng(seed)
+    V, M = 7, 20000
+    T = float(rng.choice([0.5, 1.0, 2.0]))
+    x = rng.standard_normal(V) * 2.0
+    us = (np.arange(M) + 0.5) / M
+    logits = np.broadcast_to(x, (1, M, V))
+    y = oracle.sample_target(logits, np.array([M]), us[None], T)[0]
+    assert (np.diff(y) >= 0).all()
+    want = np.exp(x / T - (x / T).max())
+    want /= want.sum()
+    got = np.bincount(y, minlength=V) / M
+    assert np.abs(got - want).max() <= 1.0 / M + 1e-12
+
+
 # ---------------------------------------------------------------- pin power
 def test_pins_catch_planted_mistakes():
     """Plant typical mistakes in oracle outputs; the checkers must object."""
