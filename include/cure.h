@@ -12,6 +12,8 @@
  *                     Sec. 3.3, 3.4         flattened repair tree + ancestor mask
  *   cure_tree_attn    Sec. 3.2, 3.4, 3.5    tree-masked GQA attention
  *   cure_accept       Sec. 3.5 Eq. (4)      target argmax + longest accepted path
+ *   cure_sample_target Sec. 2 (T > 0)       the target's sampled token per node, for
+ *                                           stochastic verification with cure_accept
  *   cure_resync_kv    Sec. 3.5, Alg. 1      write the path into the KV cache,
  *                                           realign the draft state
  *
@@ -233,6 +235,26 @@ cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k, const void
  *   diverge_depth [B]: shallowest path depth whose node is a repair node
  *                      (index > K), or -1 when branch 0 wins.
  */
+/*
+ * Stage 5, stochastic verification (temperature > 0).  Speculative decoding is
+ * lossless sampling from the target (Sec. 2); the paper's runs are greedy
+ * (Sec. 4.1), where cure_accept's argmax fills targ.  This call fills targ
+ * with samples instead, and cure_accept(target_logits = NULL, targ) then walks
+ * the tree unchanged: a child is accepted when its token equals its parent's
+ * sample.  Each sample is drawn independently of the drafted children, so the
+ * emitted tokens follow the target's distribution.
+ * For j < n_nodes[b]: targ[b][j] = the first id v with
+ *   sum_{w <= v} softmax(target_logits[b][j] / temperature)_w > u,
+ * u = uniforms[b][j] (float [B][n_max], clamped to [0, 1)), from float32
+ * partial sums: within their rounding of the exact inverse CDF, never an id
+ * of probability 0.  A row of -inf logits gives 0; rows j >= n_nodes[b] get -1.
+ * target_logits bf16 [B][n_max][vocab], 2-byte aligned; temperature > 0 and
+ * finite; 1 <= n_max <= 256.  One CTA per row.
+ */
+cure_status cure_sample_target(const void* target_logits, const float* uniforms, float temperature,
+                               int32_t batch, int32_t n_max, int32_t vocab, const int32_t* n_nodes,
+                               int32_t* targ, void* stream);
+
 cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch, int32_t n_max,
                         int32_t vocab, int32_t block, const int32_t* n_nodes, const int32_t* tok,
                         const int32_t* parent, const int32_t* depth, const uint64_t* anc,

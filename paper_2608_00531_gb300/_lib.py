@@ -19,7 +19,7 @@ DEVERR_PAGE, DEVERR_SLOT, DEVERR_NODES, DEVERR_TOKEN = 0x1, 0x2, 0x4, 0x8
 
 # every entry point the header declares
 EXPORTS = ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_tree_attn_workspace_size",
-           "cure_accept", "cure_resync_kv", "cure_device_error", "cure_status_string",
+           "cure_accept", "cure_sample_target", "cure_resync_kv", "cure_device_error", "cure_status_string",
            "cure_abi_version")
 
 
@@ -65,6 +65,7 @@ def load() -> C.CDLL:
     lib.cure_tree_attn_workspace_size.argtypes = [I32, I32, I32, C.POINTER(KVDesc)]
     lib.cure_tree_attn_workspace_size.restype = C.c_size_t
     lib.cure_accept.argtypes = [P, P, I32, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P]
+    lib.cure_sample_target.argtypes = [P, P, C.c_float, I32, I32, I32, P, P, P]
     lib.cure_resync_kv.argtypes = [I32, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
                                    C.POINTER(KVDesc), P, P, I32, I32, I32, P, P, P, P, P, P, P,
                                    P, P, P]

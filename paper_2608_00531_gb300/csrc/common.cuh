@@ -54,6 +54,11 @@ cudaError_t launch_score(const uint16_t* logits, int64_t rows, int vocab, int to
 // Target argmax over rows (b, j) with j < n_nodes[b]; other rows get -1.
 cudaError_t launch_target_argmax(const uint16_t* logits, int batch, int n_max, int vocab,
                                  const int32_t* n_nodes, int32_t* targ, cudaStream_t s);
+// Target token sampled at temperature T > 0 over rows (b, j) with j < n_nodes[b]
+// (inverse CDF with uniforms[b][j]); other rows get -1.
+cudaError_t launch_sample_target(const uint16_t* logits, const float* uniforms, float temperature,
+                                 int batch, int n_max, int vocab, const int32_t* n_nodes, int32_t* targ,
+                                 int* err, cudaStream_t s);
 
 cudaError_t launch_build_tree(const cure_tree_params& p, const int32_t* top_ids,
                               const float* margin, const int32_t* root_tok,

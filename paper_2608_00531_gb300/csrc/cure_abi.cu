@@ -83,7 +83,7 @@ using namespace cure;
 
 extern "C" {
 
-int32_t cure_abi_version(void) { return 102; }
+int32_t cure_abi_version(void) { return 103; }
 
 const char* cure_status_string(cure_status s) {
   switch (s) {
@@ -172,6 +172,21 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
                                     anc, batch, n_max, heads_q, scale, static_cast<uint16_t*>(out),
                                     workspace, device_error_word(),
                                     static_cast<cudaStream_t>(stream)));
+}
+
+cure_status cure_sample_target(const void* target_logits, const float* uniforms, float temperature,
+                               int32_t batch, int32_t n_max, int32_t vocab, const int32_t* n_nodes,
+                               int32_t* targ, void* stream) {
+  if (batch < 0 || n_max < 1 || vocab < 1 || !(temperature > 0.f && temperature <= FLT_MAX))
+    return CURE_ERR_INVALID_ARG;
+  if (n_max > kMaxNodes || (int64_t)batch * n_max > 65535) return CURE_ERR_UNSUPPORTED;
+  if (batch == 0) return CURE_OK;
+  if (!target_logits || !uniforms || !n_nodes || !targ || !aligned(target_logits, 2) ||
+      !aligned(uniforms, 4))
+    return CURE_ERR_INVALID_ARG;
+  return from_cuda(launch_sample_target(static_cast<const uint16_t*>(target_logits), uniforms, temperature,
+                                        batch, n_max, vocab, n_nodes, targ, device_error_word(),
+                                        static_cast<cudaStream_t>(stream)));
 }
 
 cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch, int32_t n_max,

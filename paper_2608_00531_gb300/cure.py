@@ -183,6 +183,23 @@ def cure_accept(tree: dict, block: int, *, target_logits: Optional[torch.Tensor]
     return out
 
 
+def cure_sample_target(target_logits: torch.Tensor, n_nodes: torch.Tensor, uniforms: torch.Tensor,
+                       temperature: float, *, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Stochastic verification (Sec. 2, T > 0): the target's token at every tree
+    node sampled by inverse CDF with uniforms[b][j]; pass the result to
+    cure_accept as ``targ`` (without target_logits) for the walk."""
+    _need(target_logits, torch.bfloat16, "target_logits")
+    _need(uniforms, torch.float32, "uniforms")
+    B, n_max, V = target_logits.shape
+    if out is None:
+        out = torch.empty(B, n_max, dtype=torch.int32, device=target_logits.device)
+    lib = _lib.load()
+    check("cure_sample_target", lib.cure_sample_target(
+        _p(target_logits), _p(uniforms), float(temperature), B, n_max, V, _p(n_nodes), _p(out),
+        _stream(stream)))
+    return out
+
+
 def cure_resync_kv(k_caches: Sequence[torch.Tensor], v_caches: Sequence[torch.Tensor], kv: KVDesc,
                    tree_k: Optional[torch.Tensor], tree_v: Optional[torch.Tensor], acc: dict,
                    cache_len_in: torch.Tensor, block: int, *, n_max: Optional[int] = None,

@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert lib.cure_abi_version() == 102
+    assert lib.cure_abi_version() == 103
     assert lib.cure_status_string(0) == b"ok"
     assert lib.cure_status_string(2) == b"workspace too small"
 
@@ -84,6 +84,12 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
         p.max_depth, p.beam = md, bw
         assert lib.cure_build_tree(C.byref(p), *([null] * 13), null) == want, (md, bw)
     p.max_depth, p.beam = 0, 0
+    # sampling: the temperature must be positive and finite; batch 0 is a no-op
+    dev = C.c_void_p(256)
+    for T, want in ((0.0, 1), (-1.0, 1), (float("inf"), 1), (float("nan"), 1)):
+        assert lib.cure_sample_target(dev, dev, C.c_float(T), 1, 9, 100, dev, dev, null) == want, T
+    assert lib.cure_sample_target(dev, null, C.c_float(1.0), 1, 9, 100, dev, dev, null) == 1
+    assert lib.cure_sample_target(null, null, C.c_float(1.0), 0, 9, 100, null, null, null) == 0
     # attention: head_dim 64 unsupported, heads_q not a multiple of heads_kv
     kv = KVDesc(layout=0, heads_kv=4, head_dim=64, page_size=16, max_len=100, num_pages=0, block_table=None)
     assert lib.cure_tree_attn(*([null] * 5), C.byref(kv), null, null, null, 1, 9, 8, 1.0, null, null, 0, null) == 5

@@ -570,6 +570,121 @@ def test_accept_random_trees_with_ids(cure, seed):
         assert np.array_equal(acc[key].cpu().numpy(), o_acc[key]), key
 
 
+# ------------------------------------------------------ stochastic verification
+def _valid_sample(x, T, u, y, tol=1e-4):
+    """y is a valid inverse-CDF draw for u: an id of nonzero probability whose
+    cumulative range (float64) contains u Z, up to float32 summation (tol Z)."""
+    m = x.max()
+    if m == -np.inf:
+        return y == 0
+    p = np.exp((x - m) / T)
+    c = np.cumsum(p)
+    Z = c[-1]
+    r = min(max(u, 0.0), float(np.nextafter(np.float32(1), np.float32(0)))) * Z
+    if not (0 <= y < len(x)) or p[y] <= 0:
+        return False
+    lo = c[y - 1] if y > 0 else 0.0
+    return lo - tol * Z <= r <= c[y] + tol * Z
+
+
+@pytest.mark.parametrize("V", [1000, 4099, 151936])
+@pytest.mark.parametrize("T", [0.5, 1.0, 2.0])
+def test_sample_target_inverse_cdf(cure, V, T):
+    rng = np.random.default_rng(V + int(10 * T))
+    B, N = 4, 9
+    n = np.array([1, 5, 9, 3], dtype=np.int32)
+    x = (rng.standard_normal((B, N, V)) * 2.0).astype(np.float32)
+    x[2, 1, :] = -np.inf
+    x[2, 1, 17] = 3.0                 # one finite logit
+    x[2, 2, :] = -np.inf              # none: id 0
+    x[3, 0, : V // 2] = -np.inf       # the first half impossible
+    logits = W.to_bf16(x)
+    u = rng.random((B, N)).astype(np.float32)
+    u[1, 0], u[1, 1], u[3, 0] = 0.0, np.float32(0.9999999), 0.0
+    got = cure.cure_sample_target(logits.to(DEV), torch.from_numpy(n).to(DEV), torch.from_numpy(u).to(DEV),
+                                  T).cpu().numpy()
+    assert cure.cure_device_error() == 0
+    xf = _f64(logits)
+    for b in range(B):
+        for j in range(N):
+            if j >= n[b]:
+                assert got[b, j] == -1
+            else:
+                assert _valid_sample(xf[b, j], T, float(u[b, j]), int(got[b, j])), (b, j, got[b, j])
+    assert got[2, 1] == 17 and got[2, 2] == 0 and got[3, 0] >= V // 2
+
+
+def test_sample_target_frequencies_follow_softmax(cure):
+    """2000 rows of the same 7 logits with u on a grid: the ids drawn match
+    the oracle's exact inverse CDF (but for u within rounding of a boundary),
+    so their frequencies are the softmax probabilities to one grid step."""
+    rng = np.random.default_rng(5)
+    B, N, V, T = 250, 8, 7, 0.7
+    x = np.broadcast_to(rng.standard_normal(V).astype(np.float32) * 2.0, (B, N, V)).copy()
+    logits = W.to_bf16(x)
+    M = B * N
+    u = ((np.arange(M) + 0.5) / M).astype(np.float32).reshape(B, N)
+    n = np.full(B, N, dtype=np.int32)
+    got = cure.cure_sample_target(logits.to(DEV), torch.from_numpy(n).to(DEV), torch.from_numpy(u).to(DEV),
+                                  T).cpu().numpy()
+    want = oracle.sample_target(_f64(logits), n, u.astype(np.float64), T)
+    assert (got != want).sum() <= 2
+    p = np.exp(_f64(logits)[0, 0] / T)
+    p /= p.sum()
+    assert np.abs(np.bincount(got.ravel(), minlength=V) / M - p).max() <= 2.0 / M
+
+
+def test_sample_target_then_accept(cure):
+    """Stochastic verification end to end: sampled target tokens, then the
+    unchanged acceptance walk, against the oracle walk on the same samples."""
+    w = W.WORKLOADS["tiny"].replace(batch=8, vocab=512)
+    rng = np.random.default_rng(9)
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, 1)
+    N = w.n_max
+    # target logits that favour the draft's tokens, so that paths get accepted
+    x = rng.standard_normal((w.batch, N, w.vocab)).astype(np.float32)
+    for b in range(w.batch):
+        for j in range(int(t["n_nodes"][b])):
+            kids = [c for c in range(int(t["n_nodes"][b])) if t["parent"][b, c] == j]
+            for c in kids:
+                x[b, j, int(t["tok"][b, c])] += 9.0
+    logits = W.to_bf16(x)
+    u = rng.random((w.batch, N)).astype(np.float32)
+    tree_d = _gpu_tree_dict(t)
+    targ = cure.cure_sample_target(logits.to(DEV), tree_d["n_nodes"], torch.from_numpy(u).to(DEV), 1.0)
+    acc = cure.cure_accept(tree_d, w.block, targ=targ)
+    g = targ.cpu().numpy()
+    xf = _f64(logits)
+    for b in range(w.batch):
+        for j in range(int(t["n_nodes"][b])):
+            assert _valid_sample(xf[b, j], 1.0, float(u[b, j]), int(g[b, j]))
+    o = oracle.accept(g, t["n_nodes"], t["tok"], t["parent"], t["depth"], t["anc"], w.block)
+    for key in ("accept_len", "best_node", "path_nodes", "out_tokens", "diverge_depth"):
+        assert np.array_equal(acc[key].cpu().numpy(), o[key]), key
+    assert o["accept_len"].max() > 0
+
+
+def test_sample_target_serving_shape_sampled(cure):
+    """The serving shape (32 x 33 rows of 151936 logits), rows checked on a sample."""
+    B, N, V = 32, 33, 151936
+    g = torch.Generator(device=DEV).manual_seed(11)
+    logits = (torch.randn(B, N, V, generator=g, device=DEV) * 3).to(torch.bfloat16)
+    n = torch.randint(17, N + 1, (B,), generator=g, device=DEV, dtype=torch.int32)
+    u = torch.rand(B, N, generator=g, device=DEV)
+    got = cure.cure_sample_target(logits, n, u, 0.8).cpu().numpy()
+    nh, uh = n.cpu().numpy(), u.cpu().numpy()
+    rng = np.random.default_rng(3)
+    for _ in range(24):
+        b, j = int(rng.integers(0, B)), int(rng.integers(0, N))
+        if j >= nh[b]:
+            assert got[b, j] == -1
+        else:
+            xr = logits[b, j].float().cpu().numpy().astype(np.float64)
+            assert _valid_sample(xr, 0.8, float(uh[b, j]), int(got[b, j])), (b, j)
+
+
 # ------------------------------------------------------------------ resync
 @pytest.mark.parametrize("paged", [0, 8, 16, 32, 64])
 def test_resync(cure, paged):
