@@ -269,7 +269,10 @@ def test_branch_budget_closed_forms():
     hand value; x = 1.5, 2.5, 3.5 and 4.5 pin the halves (away from zero:
     half to even would give 2, 2, 4, 4).
     """
-    bb = oracle.branch_budget
+    assert _branch_budget_closed_forms_hold(oracle.branch_budget)
+
+
+def _branch_budget_closed_forms_hold(bb):
     cases = [(0.0, 5),    # u = 1: a tied position gets b_max
              (2.0, 4),    # u = 3/4: x = 4
              (3.0, 4),    # u = 5/8: x = 3.5
@@ -280,13 +283,11 @@ def test_branch_budget_closed_forms():
              (1.0, 5),    # u = 7/8: x = 4.5
              (8.0, 1),    # u = 0: b_min
              (12.0, 1)]   # m > s: u clipped to 0
-    for m, want in cases:
-        assert bb(np.float32(m), 8.0, 1, 5) == want, (m, want)
-    for m in (0.0, 0.3, 7.9, 100.0):          # b_min = b_max: constant
-        assert bb(np.float32(m), 1.0, 3, 3) == 3
-    assert bb(np.float32(1.0), 1.0, 0, 4) == 0    # b_min = 0 is reachable
-    assert bb(np.float32(0.0), 1.0, 0, 4) == 4
-    assert bb(np.float32(np.inf), 1.0, 1, 5) == 1  # rival at -inf: margin +inf
+    ok = all(bb(np.float32(m), 8.0, 1, 5) == want for m, want in cases)
+    ok = ok and all(bb(np.float32(m), 1.0, 3, 3) == 3 for m in (0.0, 0.3, 7.9, 100.0))  # b_min = b_max
+    ok = ok and bb(np.float32(1.0), 1.0, 0, 4) == 0 and bb(np.float32(0.0), 1.0, 0, 4) == 4
+    ok = ok and bb(np.float32(np.inf), 1.0, 1, 5) == 1   # rival at -inf: margin +inf
+    return ok
 
 
 @pytest.mark.parametrize("seed", range(6))
@@ -739,23 +740,26 @@ def test_resync_in_place_hand(case):
 def test_sample_target_closed_forms():
     """Inverse-CDF sampling by hand: equal logits give floor(u V); two finite
     logits a, b give the first id while u < e^(a/T) / (e^(a/T) + e^(b/T))."""
+    assert _sample_closed_forms_hold(oracle.sample_target)
+
+
+def _sample_closed_forms_hold(sample):
     V = 10
     x = np.zeros((1, 1, V))
+    ok = True
     for u in (0.0, 0.05, 0.31, 0.5, 0.99):
-        y = oracle.sample_target(x, np.array([1]), np.array([[u]]), 1.0)[0, 0]
-        assert y == math.floor(u * V), (u, y)
+        ok = ok and sample(x, np.array([1]), np.array([[u]]), 1.0)[0, 0] == math.floor(u * V)
     x = np.full((1, 1, V), -np.inf)
     x[0, 0, 3], x[0, 0, 7] = 1.0, 2.0
     for T in (0.5, 1.0, 3.0):
         p3 = math.exp(1.0 / T) / (math.exp(1.0 / T) + math.exp(2.0 / T))
         for u in (0.0, p3 - 1e-9, p3 + 1e-9, 0.999):
-            y = oracle.sample_target(x, np.array([1]), np.array([[u]]), T)[0, 0]
-            assert y == (3 if u < p3 else 7), (T, u, y)
+            ok = ok and sample(x, np.array([1]), np.array([[u]]), T)[0, 0] == (3 if u < p3 else 7)
     # one finite logit: always that id; only -inf: id 0; rows past n_nodes: -1
     x = np.full((1, 3, V), -np.inf)
     x[0, 0, 6] = -4.0
-    y = oracle.sample_target(x, np.array([2]), np.array([[0.7, 0.2, 0.5]]), 1.0)
-    assert y[0].tolist() == [6, 0, -1]
+    y = sample(x, np.array([2]), np.array([[0.7, 0.2, 0.5]]), 1.0)
+    return bool(ok and y[0].tolist() == [6, 0, -1])
 
 
 @pytest.mark.parametrize("seed", range(4))
@@ -778,6 +782,56 @@ def test_sample_target_frequencies_follow_softmax(seed):
 
 
 # ---------------------------------------------------------------- pin power
+def test_new_pins_catch_planted_mistakes():
+    """Mutants of Eq. (3) and of the inverse-CDF sampler, each a plausible
+    slip; the closed-form checkers must reject every one."""
+    f = np.float32
+
+    def bb_half_even(m, s, lo, hi):          # round() half to even
+        u = f(min(max(f(f(1) - f(f(m) / f(s))), f(0)), f(1)))
+        x = f(f(lo) + f(u * f(hi - lo)))
+        return int(min(max(int(np.rint(x)), lo), hi))
+
+    def bb_swapped(m, s, lo, hi):            # b_min and b_max exchanged
+        return oracle.branch_budget(m, s, hi, lo) if hi >= lo else lo
+
+    def bb_no_complement(m, s, lo, hi):      # u = m / s instead of 1 - m / s
+        u = f(min(max(f(f(m) / f(s)), f(0)), f(1)))
+        x = f(f(lo) + f(u * f(hi - lo)))
+        return int(min(max(math.floor(float(x) + 0.5), lo), hi))
+
+    def bb_branches_not_alternatives(m, s, lo, hi):   # b_i counting the draft token too
+        return max(lo, oracle.branch_budget(m, s, lo, hi) - 1)
+
+    assert _branch_budget_closed_forms_hold(oracle.branch_budget)
+    for mutant in (bb_half_even, bb_swapped, bb_no_complement, bb_branches_not_alternatives):
+        assert not _branch_budget_closed_forms_hold(mutant), mutant.__name__
+
+    def sample_left(logits, n_nodes, uniforms, T):     # first id with cumulative >= r
+        out = np.full(logits.shape[:2], -1, dtype=np.int64)
+        for b in range(logits.shape[0]):
+            for j in range(int(n_nodes[b])):
+                x = logits[b, j]
+                if x.max() == -np.inf:
+                    out[b, j] = 0
+                    continue
+                c = np.cumsum(np.exp((x - x.max()) / T))
+                out[b, j] = int(np.searchsorted(c, uniforms[b, j] * c[-1], side="left"))
+        return out
+
+    def sample_times_T(logits, n_nodes, uniforms, T):  # logits scaled by T, not by 1/T
+        return oracle.sample_target(logits, n_nodes, uniforms, 1.0 / T)
+
+    def sample_no_mask(logits, n_nodes, uniforms, T):  # -inf rows not special-cased, tail not -1
+        y = oracle.sample_target(np.where(np.isinf(logits), -30.0, logits), np.full_like(n_nodes, logits.shape[1]),
+                                 uniforms, T)
+        return y
+
+    assert _sample_closed_forms_hold(oracle.sample_target)
+    for mutant in (sample_left, sample_times_T, sample_no_mask):
+        assert not _sample_closed_forms_hold(mutant), mutant.__name__
+
+
 def test_pins_catch_planted_mistakes():
     """Plant typical mistakes in oracle outputs; the checkers must object."""
     top, margin, root, L, tau, budget, branches, d, redraft = _random_case(4, K=8, budget=5, tau=2.0,
