@@ -832,6 +832,39 @@ def test_new_pins_catch_planted_mistakes():
         assert not _sample_closed_forms_hold(mutant), mutant.__name__
 
 
+def test_cap_and_in_place_pins_catch_planted_mistakes(monkeypatch):
+    """A depth cap that drops the whole alternative (not only its successor)
+    and an in-place layout read one slot late must fail their pins."""
+    import oracle.cure_oracle as oc
+    real_cost = oc.repair_cost
+
+    def cost_drops_alternative(i, K, repair_depth, max_depth=0):
+        c = min(repair_depth, K - i)
+        return 0 if (max_depth > 0 and i + c > max_depth) else c
+
+    monkeypatch.setattr(oc, "repair_cost", cost_drops_alternative)
+    t = _caps_hand(d=2, max_depth=2)
+    assert t["n_nodes"][0] != 5 + 6            # the hand pin expects six repair nodes
+    monkeypatch.setattr(oc, "repair_cost", real_cost)
+    assert _caps_hand(d=2, max_depth=2)["n_nodes"][0] == 5 + 6
+
+    real_rows = oc.tree_rows_in_cache
+
+    def rows_one_late(cache, cache_len, n_nodes, N, block_table, page_size):
+        return real_rows(cache, np.asarray(cache_len) + 1, n_nodes, N, block_table, page_size)
+
+    q, tk, tv, kc, vc, L, t, D = _attn_case(0)
+    ck, cv, _ = _in_place_caches(kc, vc, tk, tv, L, t["n_nodes"], False)
+    ck = np.concatenate([ck, np.zeros_like(ck[:, :1])], axis=1)   # room for the late read
+    cv = np.concatenate([cv, np.zeros_like(cv[:, :1])], axis=1)
+    good = oracle.tree_attn(q, None, None, ck, cv, L, t["n_nodes"], t["anc"], 1.0 / math.sqrt(D))
+    sep = oracle.tree_attn(q, tk, tv, kc, vc, L, t["n_nodes"], t["anc"], 1.0 / math.sqrt(D))
+    monkeypatch.setattr(oc, "tree_rows_in_cache", rows_one_late)
+    bad = oracle.tree_attn(q, None, None, ck, cv, L, t["n_nodes"], t["anc"], 1.0 / math.sqrt(D))
+    assert np.allclose(good, sep, rtol=1e-12, atol=1e-13)
+    assert not np.allclose(bad, sep, rtol=1e-6, atol=1e-6)
+
+
 def test_pins_catch_planted_mistakes():
     """Plant typical mistakes in oracle outputs; the checkers must object."""
     top, margin, root, L, tau, budget, branches, d, redraft = _random_case(4, K=8, budget=5, tau=2.0,
