@@ -4,8 +4,8 @@
  * CURE ("Local Uncertainty Repair for Block-Parallel Speculative Decoding")
  * repairs a block-parallel draft at its low-margin positions and verifies the
  * draft and the repairs in one tree pass.  One decoding step of the method is
- * split into five calls, each one CUDA kernel (or two) on the caller's
- * stream:
+ * split into five calls (a sixth replaces the greedy argmax when verifying at
+ * a temperature), each one CUDA kernel (or two) on the caller's stream:
  *
  *   cure_score_draft  Sec. 3.3, Eq. (2)     top-k ids, margin, top-1 log-prob
  *   cure_build_tree   Sec. 3.1 Eq. (1),     UFP gate + budgeted selection,
