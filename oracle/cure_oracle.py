@@ -15,6 +15,8 @@ Stages and the passages they follow:
                    construction, branch 0 anchored)
 * ``tree_attn``    Sec. 3.2 / 3.4 / 3.5 (single-pass Tree Attention)
 * ``accept``       Sec. 3.5 Eq. (4) with greedy decoding (Sec. 4.1)
+* ``lm_head_argmax`` the target's greedy token per node from its final
+                   hidden state and the LM-head weight (Sec. 3.5, Sec. 4.1)
 * ``sample_target`` the target's token per node at a temperature T > 0
                    (Sec. 2: lossless speculative sampling; the paper's own
                    runs are greedy, Sec. 4.1)
@@ -109,6 +111,29 @@ def row_argmax(logits: np.ndarray) -> np.ndarray:
     for r in range(x.shape[0]):
         out[r] = int(np.argmax(x[r]))      # numpy returns the first maximum
     return out
+
+
+def lm_head_argmax(hidden: np.ndarray, w_lm: np.ndarray) -> np.ndarray:
+    """The target's greedy token at each tree node from its final hidden state
+    (Sec. 3.5, Eq. 4: the target scores every node in one pass; greedy
+    decoding, Sec. 4.1): the first maximum over v of the logit
+    hidden[r] . w_lm[v], all in float64.
+
+    ``hidden`` is [rows][d_model] and ``w_lm`` the LM-head weight [vocab][d_model],
+    both holding bf16 values widened exactly; every product of two bf16 values
+    is exact in float64, so the logits are the exact dot products up to float64
+    summation.  The fused kernel never writes these logits; its argmax must
+    match this one wherever the float32 accumulation bound cannot reorder the
+    top two.
+    """
+    h = np.asarray(hidden, dtype=np.float64)
+    V = w_lm.shape[0]
+    # the logits [rows][vocab], computed over slices of the vocabulary only to
+    # bound the float64 copy of the weight held at once
+    chunk = 8192
+    logits = np.concatenate([h @ np.asarray(w_lm[v0:v0 + chunk], dtype=np.float64).T
+                             for v0 in range(0, V, chunk)], axis=1)
+    return row_argmax(logits)
 
 
 # --------------------------------------------------------------------------

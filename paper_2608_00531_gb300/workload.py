@@ -238,3 +238,35 @@ def block_table(cache_len: np.ndarray, block: int, seed: int,
 
 def normal_bf16(shape, std: float, rng: np.random.Generator) -> torch.Tensor:
     return to_bf16(rng.standard_normal(shape, dtype=np.float32) * np.float32(std))
+
+
+# ------------------------------------------------------------------ LM head
+def lm_head_weight(vocab: int, d_model: int, seed: int, chunk: int = 16384) -> torch.Tensor:
+    """A seeded stand-in for the target's LM-head weight, bf16 [vocab][d_model]:
+    N(0, 1/d_model) entries, so each row's squared norm is about 1.  Drawn in
+    slices of the vocabulary (each slice from its own seeded stream) to bound
+    the float32 memory held at once."""
+    out = torch.empty(vocab, d_model, dtype=torch.bfloat16)
+    sd = np.float32(1.0 / np.sqrt(d_model))
+    for i, v0 in enumerate(range(0, vocab, chunk)):
+        rng = np.random.default_rng([seed, 7717, i])
+        n = min(chunk, vocab - v0)
+        out[v0:v0 + n] = to_bf16(rng.standard_normal((n, d_model), dtype=np.float32) * sd)
+    return out
+
+
+def lm_head_hidden(rows: int, w_lm: torch.Tensor, seed: int, planted: Optional[np.ndarray] = None,
+                   strength: float = 12.0) -> torch.Tensor:
+    """Seeded final hidden states bf16 [rows][d_model]: N(0, 1) entries, plus
+    ``strength`` times the weight row of ``planted[r]`` where planted[r] >= 0,
+    so that logit's expected value is about ``strength`` against N(0, 1) for the
+    others (a stand-in target that prefers the planted token)."""
+    d = w_lm.shape[1]
+    rng = np.random.default_rng([seed, 4243])
+    h = rng.standard_normal((rows, d), dtype=np.float32)
+    if planted is not None:
+        sel = np.flatnonzero(np.asarray(planted) >= 0)
+        if len(sel):
+            wt = w_lm[torch.from_numpy(np.asarray(planted)[sel].astype(np.int64))].to(torch.float32).numpy()
+            h[sel] += np.float32(strength) * wt
+    return to_bf16(h)

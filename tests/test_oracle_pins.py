@@ -893,3 +893,90 @@ def test_pins_catch_planted_mistakes():
     m32 = np.full((1, 4), 1.0, dtype=np.float32)
     t_le = oracle.build_tree(top[:1, :4], m32 - np.float32(1e-7), root[:1], L[:1], 1.0, 8, 2, 1)
     assert check_tree(t_le, top[:1, :4], m32, 1.0, 8, 2, 1, L[:1]) != []
+
+
+# ---------------------------------------------------------------- LM-head argmax pins
+def _lm_bruteforce(h, w):
+    """Every logit as an exactly rounded sum (math.fsum) of its products, then
+    the first maximum by a scan: the definition with no library matmul."""
+    out = []
+    for r in range(h.shape[0]):
+        best, bi = None, -1
+        for v in range(w.shape[0]):
+            s = math.fsum(float(h[r, k]) * float(w[v, k]) for k in range(h.shape[1]))
+            if best is None or s > best:
+                best, bi = s, v
+        out.append(bi)
+    return np.array(out)
+
+
+def _lm_case(seed, rows=6, V=41, d=12):
+    rng = np.random.default_rng(seed)
+    h = W.bf16_to_f64(W.to_bf16(rng.standard_normal((rows, d)).astype(np.float32)))
+    w = W.bf16_to_f64(W.to_bf16(rng.standard_normal((V, d)).astype(np.float32)))
+    w[7] = w[3]                        # two identical rows: ties between ids 3 and 7
+    h[0] = w[3] * 4.0                  # row 0 prefers that direction
+    return h, w
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_lm_head_argmax_bruteforce(seed):
+    h, w = _lm_case(seed)
+    got = oracle.lm_head_argmax(h, w)
+    assert np.array_equal(got, _lm_bruteforce(h, w))
+    assert got[0] == 3                 # the tie between 3 and 7 goes to the lower id
+
+
+def test_lm_head_argmax_basis_rows_and_square_shape():
+    """hidden = c e_k picks the first maximum (c > 0) or first minimum (c < 0)
+    of the weight's column k; a square weight, whose transpose has the same
+    shape, tells w from w^T."""
+    rng = np.random.default_rng(3)
+    d = 9
+    w = W.bf16_to_f64(W.to_bf16(rng.standard_normal((d, d)).astype(np.float32)))
+    for k in range(d):
+        for c in (1.0, -2.0):
+            h = np.zeros((1, d))
+            h[0, k] = c
+            col = w[:, k] * c
+            assert oracle.lm_head_argmax(h, w)[0] == int(np.flatnonzero(col == col.max())[0])
+    h = W.bf16_to_f64(W.to_bf16(rng.standard_normal((5, d)).astype(np.float32)))
+    assert np.array_equal(oracle.lm_head_argmax(h, w), _lm_bruteforce(h, w))
+    assert not np.array_equal(_lm_bruteforce(h, w.T), _lm_bruteforce(h, w))
+
+
+def test_lm_head_argmax_planted_stand_in_target():
+    """The synthetic hidden states built from a planted token give that token,
+    at the serving vocabulary with a small model width (the construction's
+    logit margin is about 12 against N(0, 1) noise)."""
+    w = W.lm_head_weight(151936, 128, 11)
+    planted = np.array([0, 151935, 5, -1, 77777, 5])
+    h = W.lm_head_hidden(6, w, 11, planted, strength=40.0)
+    got = oracle.lm_head_argmax(W.bf16_to_f64(h), w.to(torch.float32).numpy())
+    sel = planted >= 0
+    assert np.array_equal(got[sel], planted[sel])
+
+
+def test_lm_head_pins_catch_planted_mistakes():
+    """A transposed weight, a last-maximum tie rule and a dropped feature must
+    each fail the brute-force or tie pins."""
+    h, w = _lm_case(0, rows=5, V=12, d=12)
+    good = _lm_bruteforce(h, w)
+
+    def transposed(h, w):
+        return oracle.lm_head_argmax(h, w.T)
+
+    def last_max(h, w):
+        lg = h @ w.T
+        return np.array([len(r) - 1 - int(np.argmax(r[::-1])) for r in lg])
+
+    def dropped_feature(h, w):
+        return oracle.lm_head_argmax(h[:, :-1], w[:, :-1])
+
+    h2 = h.copy()
+    h2[1:, -1] *= 64.0                  # the last feature decides rows 1..4
+    good2 = _lm_bruteforce(h2, w)
+    assert np.array_equal(oracle.lm_head_argmax(h, w), good)
+    assert not np.array_equal(transposed(h, w), good)
+    assert last_max(h, w)[0] == 7 and good[0] == 3
+    assert not np.array_equal(dropped_feature(h2, w), good2)
