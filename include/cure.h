@@ -12,6 +12,8 @@
  *                     Sec. 3.3, 3.4         flattened repair tree + ancestor mask
  *   cure_tree_attn    Sec. 3.2, 3.4, 3.5    tree-masked GQA attention
  *   cure_accept       Sec. 3.5 Eq. (4)      target argmax + longest accepted path
+ *   cure_lm_head_argmax Sec. 3.5, 4.1       the target's argmax per node straight from
+ *                                           its hidden state (LM head + argmax fused)
  *   cure_sample_target Sec. 2 (T > 0)       the target's sampled token per node, for
  *                                           stochastic verification with cure_accept
  *   cure_resync_kv    Sec. 3.5, Alg. 1      write the path into the KV cache,
@@ -247,13 +249,46 @@ cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k, const void
  *   sum_{w <= v} softmax(target_logits[b][j] / temperature)_w > u,
  * u = uniforms[b][j] (float [B][n_max], clamped to [0, 1)), from float32
  * partial sums: within their rounding of the exact inverse CDF, never an id
- * of probability 0.  A row of -inf logits gives 0; rows j >= n_nodes[b] get -1.
- * target_logits bf16 [B][n_max][vocab], 2-byte aligned; temperature > 0 and
- * finite; 1 <= n_max <= 256.  One CTA per row.
+ * of probability 0.  The probabilities are formed as 2^((l - l_max) log2(e)/T),
+ * which cannot overflow: at temperatures so small that every logit below the
+ * maximum underflows, the draw picks among the ids that hold the maximum
+ * (the limit T -> 0).  A row of -inf logits gives 0; rows j >= n_nodes[b]
+ * get -1.  target_logits bf16 [B][n_max][vocab], 2-byte aligned; temperature
+ * > 0 with log2(e)/temperature finite (T >= about 4.2e-39, else
+ * CURE_ERR_INVALID_ARG); 1 <= n_max <= 256.  One CTA of four warps per row,
+ * each warp streaming a contiguous quarter of it.
  */
 cure_status cure_sample_target(const void* target_logits, const float* uniforms, float temperature,
                                int32_t batch, int32_t n_max, int32_t vocab, const int32_t* n_nodes,
                                int32_t* targ, void* stream);
+
+/*
+ * Stage 5 fused with the target's LM head (Sec. 3.5, Eq. 4: the target scores
+ * every tree node in one pass; greedy decoding, Sec. 4.1).  For each of `rows`
+ * final hidden states (the tree nodes of all sequences, packed):
+ *   targ[out_index ? out_index[r] : r] = the first v maximising hidden[r] . w_lm[v]
+ * The contraction runs on the tensor cores with float32 accumulation and the
+ * argmax is taken in its epilogue: the rows x vocab logits are never written.
+ * Two ids whose logits lie within float32 accumulation error of each other may
+ * be ranked either way (d_model products per logit; the bound is about
+ * d_model/16 roundings of 2^-23 relative to sum_k |hidden[r][k] w_lm[v][k]|).
+ * Then call cure_accept(target_logits = NULL, targ).
+ * hidden: bf16 [rows][d_model]; w_lm: bf16 [vocab][d_model] (row-major, the
+ * layout of an LM-head weight); both 16-byte aligned.  d_model a multiple of
+ * 64 (else CURE_ERR_UNSUPPORTED).  out_index: int32 [rows] (NULL: identity),
+ * e.g. b * n_max + j to fill cure_accept's targ [B][n_max] from rows packed over
+ * the valid nodes; entries of targ that no row maps to are left unwritten.
+ * workspace: at least cure_lm_head_workspace_size(rows, vocab) bytes (computed
+ * for the current device), 256-byte aligned, contents on entry do not matter;
+ * calls that can overlap on the GPU must not share one.  Two kernels: the
+ * persistent tcgen05 contraction (one CTA per SM) and a per-row merge.
+ */
+cure_status cure_lm_head_argmax(const void* hidden, const void* w_lm, int32_t rows, int32_t d_model,
+                                int32_t vocab, const int32_t* out_index, int32_t* targ, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace cure_lm_head_argmax needs on the current device (0 on a bad argument). */
+size_t cure_lm_head_workspace_size(int32_t rows, int32_t vocab);
 
 cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch, int32_t n_max,
                         int32_t vocab, int32_t block, const int32_t* n_nodes, const int32_t* tok,

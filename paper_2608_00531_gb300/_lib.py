@@ -19,7 +19,7 @@ DEVERR_PAGE, DEVERR_SLOT, DEVERR_NODES, DEVERR_TOKEN = 0x1, 0x2, 0x4, 0x8
 
 # every entry point the header declares
 EXPORTS = ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_tree_attn_workspace_size",
-           "cure_accept", "cure_sample_target", "cure_resync_kv", "cure_device_error", "cure_status_string",
+           "cure_accept", "cure_lm_head_argmax", "cure_lm_head_workspace_size", "cure_sample_target", "cure_resync_kv", "cure_device_error", "cure_status_string",
            "cure_abi_version")
 
 
@@ -66,6 +66,9 @@ def load() -> C.CDLL:
     lib.cure_tree_attn_workspace_size.restype = C.c_size_t
     lib.cure_accept.argtypes = [P, P, I32, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, P]
     lib.cure_sample_target.argtypes = [P, P, C.c_float, I32, I32, I32, P, P, P]
+    lib.cure_lm_head_argmax.argtypes = [P, P, I32, I32, I32, P, P, P, C.c_size_t, P]
+    lib.cure_lm_head_workspace_size.argtypes = [I32, I32]
+    lib.cure_lm_head_workspace_size.restype = C.c_size_t
     lib.cure_resync_kv.argtypes = [I32, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
                                    C.POINTER(KVDesc), P, P, I32, I32, I32, P, P, P, P, P, P, P,
                                    P, P, P]
@@ -74,7 +77,7 @@ def load() -> C.CDLL:
     lib.cure_status_string.restype = C.c_char_p
     lib.cure_abi_version.restype = I32
     for name in ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_accept",
-                 "cure_resync_kv", "cure_device_error"):
+                 "cure_resync_kv", "cure_device_error", "cure_sample_target", "cure_lm_head_argmax"):
         getattr(lib, name).restype = C.c_int
     _lib = lib
     return lib

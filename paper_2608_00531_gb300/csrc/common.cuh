@@ -16,6 +16,15 @@ constexpr int kAttnBatchLimit = 256;  // tree attention: sequences per call
 int* device_error_word();
 int num_sms();
 
+// Device address of a __device__ variable of this library in the current
+// device's current context.  The address belongs to the context (a reset or
+// a re-created primary context gets a new one), so the cache is keyed by the
+// driver's unique context id, and looked up again whenever that id changes or
+// cannot be read.  `symbol` is the variable's host-side stand-in.
+struct SymbolCache;
+SymbolCache* new_symbol_cache();
+cudaError_t device_symbol_address(SymbolCache* cache, const void* symbol, void** out);
+
 __device__ __forceinline__ void flag(int* err, int bits) {
   if (err) atomicOr(err, bits);
 }
@@ -85,6 +94,17 @@ cudaError_t launch_resync(int layers, const LayerPtrs& caches, const cure_kv_des
                           const int32_t* cache_len_in, int32_t* cache_len_out,
                           int32_t* draft_valid_len, int32_t* replay_tokens, int32_t* n_replay,
                           int* err, cudaStream_t s);
+
+// Fused LM head + argmax: launch plan for a shape (persistent CTAs, one
+// 128-row M tile each, vocab N tiles of 256 split into `groups` ranges).
+struct LmPlan {
+  int m_tiles = 0, n_tiles = 0, groups = 0;
+  size_t ws_bytes = 0;  // per-range (max, id) partials: groups * rows * 8 bytes
+};
+LmPlan plan_lm_head(int rows, int vocab);
+cudaError_t launch_lm_head_argmax(const LmPlan& p, const uint16_t* hidden, const uint16_t* w_lm, int rows, int d,
+                                  int vocab, int32_t* out, const int32_t* out_index, void* workspace, int* err,
+                                  cudaStream_t s);
 
 // Tree attention: workspace layout for a shape.
 struct AttnPlan {

@@ -1,5 +1,6 @@
 // The C ABI (include/cure.h): host-side argument checks, then the launches.
 // Nothing here allocates device memory.
+#include <cuda.h>
 #include <float.h>
 #include <mutex>
 
@@ -10,12 +11,8 @@ namespace {
 
 __device__ int g_err_word;  // device error word, one per device that loads the library
 
-struct DevState {
-  int sms = 0;
-  int* err = nullptr;
-};
 std::mutex g_mu;
-DevState g_dev[64];
+int g_sms[64];
 
 int current_device() {
   int d = 0;
@@ -54,27 +51,84 @@ bool kv_ok(const cure_kv_desc* kv, cure_status* why) {
 
 }  // namespace
 
-int* device_error_word() {
-  const int d = current_device();
-  std::lock_guard<std::mutex> lk(g_mu);
-  if (!g_dev[d].err) {
+// ---- context-keyed device addresses of the library's __device__ variables
+namespace {
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+CtxGetCurrentFn g_ctx_get_current = nullptr;
+CtxGetIdFn g_ctx_get_id = nullptr;
+std::once_flag g_ctx_once;
+
+// The driver's id of the calling thread's current context; false when there
+// is none or it cannot be read (the caller then does not cache).
+bool current_context_id(unsigned long long* id) {
+  std::call_once(g_ctx_once, [] {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_err_word) != cudaSuccess) return nullptr;
-    g_dev[d].err = static_cast<int*>(p);
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_ctx_get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_ctx_get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  if (!g_ctx_get_current || !g_ctx_get_id) return false;
+  CUcontext c = nullptr;
+  if (g_ctx_get_current(&c) != CUDA_SUCCESS || !c) return false;
+  return g_ctx_get_id(c, id) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+struct SymbolCache {
+  std::mutex mu;
+  unsigned long long ctx[64] = {};
+  void* ptr[64] = {};
+};
+
+SymbolCache* new_symbol_cache() { return new SymbolCache(); }
+
+cudaError_t device_symbol_address(SymbolCache* cache, const void* symbol, void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  unsigned long long id = 0;
+  const bool have_id = current_context_id(&id);
+  std::lock_guard<std::mutex> lk(cache->mu);
+  if (have_id && cache->ptr[dev] && cache->ctx[dev] == id) {
+    *out = cache->ptr[dev];
+    return cudaSuccess;
   }
-  return g_dev[d].err;
+  void* p = nullptr;
+  e = cudaGetSymbolAddress(&p, symbol);  // loads the module into the context if needed
+  if (e != cudaSuccess) return e;
+  // the look-up may have created the context: read its id again
+  cache->ptr[dev] = current_context_id(&id) ? p : nullptr;
+  cache->ctx[dev] = id;
+  *out = p;
+  return cudaSuccess;
+}
+
+int* device_error_word() {
+  static SymbolCache* cache = new_symbol_cache();
+  void* p = nullptr;
+  if (device_symbol_address(cache, &g_err_word, &p) != cudaSuccess) return nullptr;
+  return static_cast<int*>(p);
 }
 
 int num_sms() {
   const int d = current_device();
   std::lock_guard<std::mutex> lk(g_mu);
-  if (!g_dev[d].sms) {
+  if (!g_sms[d]) {
     int v = 0;
     if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d) != cudaSuccess || v <= 0)
       v = 148;
-    g_dev[d].sms = v;
+    g_sms[d] = v;
   }
-  return g_dev[d].sms;
+  return g_sms[d];
 }
 
 }  // namespace cure
@@ -83,7 +137,7 @@ using namespace cure;
 
 extern "C" {
 
-int32_t cure_abi_version(void) { return 103; }
+int32_t cure_abi_version(void) { return 104; }
 
 const char* cure_status_string(cure_status s) {
   switch (s) {
@@ -177,7 +231,9 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
 cure_status cure_sample_target(const void* target_logits, const float* uniforms, float temperature,
                                int32_t batch, int32_t n_max, int32_t vocab, const int32_t* n_nodes,
                                int32_t* targ, void* stream) {
-  if (batch < 0 || n_max < 1 || vocab < 1 || !(temperature > 0.f && temperature <= FLT_MAX))
+  // log2(e) / T must be a finite float: T from about 4.2e-39 up
+  if (batch < 0 || n_max < 1 || vocab < 1 || !(temperature > 0.f && temperature <= FLT_MAX) ||
+      !(1.4426950408889634f / temperature <= FLT_MAX))
     return CURE_ERR_INVALID_ARG;
   if (n_max > kMaxNodes || (int64_t)batch * n_max > 65535) return CURE_ERR_UNSUPPORTED;
   if (batch == 0) return CURE_OK;
@@ -187,6 +243,29 @@ cure_status cure_sample_target(const void* target_logits, const float* uniforms,
   return from_cuda(launch_sample_target(static_cast<const uint16_t*>(target_logits), uniforms, temperature,
                                         batch, n_max, vocab, n_nodes, targ, device_error_word(),
                                         static_cast<cudaStream_t>(stream)));
+}
+
+size_t cure_lm_head_workspace_size(int32_t rows, int32_t vocab) {
+  if (rows < 0 || vocab < 1) return 0;
+  if (rows == 0) return 256;
+  return plan_lm_head(rows, vocab).ws_bytes;
+}
+
+cure_status cure_lm_head_argmax(const void* hidden, const void* w_lm, int32_t rows, int32_t d_model,
+                                int32_t vocab, const int32_t* out_index, int32_t* targ, void* workspace,
+                                size_t workspace_bytes, void* stream) {
+  if (rows < 0 || d_model < 64 || vocab < 1) return CURE_ERR_INVALID_ARG;
+  if (d_model % 64 != 0) return CURE_ERR_UNSUPPORTED;
+  if (rows == 0) return CURE_OK;
+  if (!hidden || !w_lm || !targ || !workspace || !aligned(hidden, 16) || !aligned(w_lm, 16) ||
+      !aligned(workspace, 256) || !aligned(targ, 4) || !aligned(out_index, 4))
+    return CURE_ERR_INVALID_ARG;
+  const LmPlan plan = plan_lm_head(rows, vocab);
+  if (workspace_bytes < plan.ws_bytes) return CURE_ERR_CAPACITY;
+  return from_cuda(launch_lm_head_argmax(plan, static_cast<const uint16_t*>(hidden),
+                                         static_cast<const uint16_t*>(w_lm), rows, d_model, vocab, targ,
+                                         out_index, workspace, device_error_word(),
+                                         static_cast<cudaStream_t>(stream)));
 }
 
 cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch, int32_t n_max,

@@ -12,37 +12,18 @@
 // The array below is CURE_NOALLOC_SCRATCH_BYTES (64 MiB).  Every GPU on which
 // this part of the library is loaded keeps it until the process exits.  In
 // host code `g_attn_scratch` is only a host-side stand-in for the symbol, not
-// a device address, so its device address is looked up once per device with
-// cudaGetSymbolAddress and that address is what the kernels receive.
+// a device address: its device address is looked up with
+// cudaGetSymbolAddress, with the device current, the first time a call runs
+// in a given CUDA context, and that address is what the kernels receive.  The
+// address is cached per device and keyed by the context's id, so a context
+// that is reset and created again is looked up afresh.
 #include <float.h>
-#include <mutex>
 
 #include "common.cuh"
 
 namespace {
 
 static __device__ __align__(256) unsigned char g_attn_scratch[CURE_NOALLOC_SCRATCH_BYTES];
-
-std::mutex g_scratch_mu;
-void* g_scratch_ptr[64];  // device address of g_attn_scratch, per device ordinal
-
-// Looks up (once per device, with that device current) the device address of
-// the scratch array.
-cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lk(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_attn_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev] = p;
-  }
-  *out = g_scratch_ptr[dev];
-  return cudaSuccess;
-}
 
 }  // namespace
 
@@ -83,11 +64,14 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
   if (!plan_tree_attn(batch, n_max, heads_q, *kv, &plan)) return CURE_ERR_INVALID_ARG;
   // the shape's split-KV partials must fit in the static array
   if (plan.total() > (size_t)CURE_NOALLOC_SCRATCH_BYTES) return CURE_ERR_CAPACITY;
+  static SymbolCache* cache = new_symbol_cache();
   void* scratch = nullptr;
-  if (scratch_address(&scratch) != cudaSuccess) return CURE_ERR_CUDA;
-  // The call zeroes the piece counters at the front of the scratch itself (an
-  // asynchronous memset on the stream); every partial that is read back was
-  // written earlier in the same call.
+  if (device_symbol_address(cache, g_attn_scratch, &scratch) != cudaSuccess) return CURE_ERR_CUDA;
+  // Nothing in the array is cleared.  Its front holds the split units' piece
+  // counters: every launch tags its counter words with a fresh launch number,
+  // a word carrying another launch's tag counts as zero, and a unit whose
+  // pieces have all arrived writes zero back.  Every partial result that is
+  // read back was written earlier in the same launch.
   const cudaError_t e = launch_tree_attn(
       plan, static_cast<const uint16_t*>(q), static_cast<const uint16_t*>(tree_k),
       static_cast<const uint16_t*>(tree_v), static_cast<const uint16_t*>(k_cache),

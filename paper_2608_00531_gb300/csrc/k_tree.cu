@@ -248,6 +248,16 @@ accept_walk_kernel(int batch, int n_max, int block, const int32_t* __restrict__ 
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) bestkey = max(bestkey, __shfl_xor_sync(kFull, bestkey, off));
+  if (bestkey < 0) {
+    // no node qualified: only a corrupt root depth gets here (the root is
+    // always accepted); fall back to the root so every store below stays in
+    // the sequence's own rows
+    if (lane == 0) {
+      flag(err, CURE_DEVERR_NODES);
+      path_nodes[(int64_t)b * (block + 2)] = 0;
+    }
+    bestkey = 0xffff;
+  }
   const int best = 0xffff - (bestkey & 0xffff);
   const int a = bestkey >> 16;
 

@@ -200,6 +200,37 @@ def cure_sample_target(target_logits: torch.Tensor, n_nodes: torch.Tensor, unifo
     return out
 
 
+def cure_lm_head_workspace_size(rows: int, vocab: int) -> int:
+    return int(_lib.load().cure_lm_head_workspace_size(rows, vocab))
+
+
+def cure_lm_head_argmax(hidden: torch.Tensor, w_lm: torch.Tensor, *, out_index: Optional[torch.Tensor] = None,
+                        out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                        stream=None) -> torch.Tensor:
+    """Stage 5 fused with the LM head (Sec. 3.5, Sec. 4.1): the first argmax of
+    hidden[r] . w_lm[v] over v for every row, without writing the logits.
+
+    hidden bf16 [rows][d_model], w_lm bf16 [vocab][d_model].  ``out_index``
+    (int32 [rows]) places row r at out.view(-1)[out_index[r]]; without it the
+    result is int32 [rows].
+    """
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(w_lm, torch.bfloat16, "w_lm")
+    rows, d = hidden.shape
+    V = w_lm.shape[0]
+    dev = hidden.device
+    if out is None:
+        out = torch.empty(rows, dtype=torch.int32, device=dev)
+    lib = _lib.load()
+    ws = int(lib.cure_lm_head_workspace_size(rows, V))
+    if workspace is None or workspace.numel() < ws:
+        workspace = torch.empty(max(ws, 256), dtype=torch.uint8, device=dev)
+    check("cure_lm_head_argmax", lib.cure_lm_head_argmax(
+        _p(hidden), _p(w_lm), rows, d, V, _p(out_index), _p(out), _p(workspace), workspace.numel(),
+        _stream(stream)))
+    return out
+
+
 def cure_resync_kv(k_caches: Sequence[torch.Tensor], v_caches: Sequence[torch.Tensor], kv: KVDesc,
                    tree_k: Optional[torch.Tensor], tree_v: Optional[torch.Tensor], acc: dict,
                    cache_len_in: torch.Tensor, block: int, *, n_max: Optional[int] = None,

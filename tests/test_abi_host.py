@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert lib.cure_abi_version() == 103
+    assert lib.cure_abi_version() == 104
     assert lib.cure_status_string(0) == b"ok"
     assert lib.cure_status_string(2) == b"workspace too small"
 
@@ -148,3 +148,64 @@ def test_product_path_has_no_cpu_fallback():
     finally:
         _lib.LIB_PATH = real
         _lib._lib = saved
+
+
+def test_noalloc_rejects_shapes_beyond_its_scratch_on_the_host(lib):
+    """cure_tree_attn_noalloc returns CURE_ERR_CAPACITY for a shape whose
+    split-KV workspace exceeds its 64 MiB static array, before any CUDA call.
+    The pointers are stand-ins that are never dereferenced; the test runs only
+    where no GPU can be reached, so that a regression in the check can never
+    launch a kernel on them."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("runs only without a reachable GPU")
+    from paper_2608_00531_gb300._lib import KVDesc
+    P, I32 = C.c_void_p, C.c_int32
+    lib.cure_tree_attn_noalloc.argtypes = [P, P, P, P, P, C.POINTER(KVDesc), P, P, P, I32, I32, I32,
+                                           C.c_float, P, P]
+    lib.cure_tree_attn_noalloc.restype = C.c_int
+    fake = C.c_void_p(1 << 20)           # aligned, never dereferenced on the host
+    kv = KVDesc(layout=1, heads_kv=4, head_dim=128, page_size=16, max_len=600, num_pages=4096,
+                block_table=fake)
+    scratch = 64 * 1024 * 1024
+    assert lib.cure_tree_attn_workspace_size(200, 33, 28, C.byref(kv)) > scratch
+    assert lib.cure_tree_attn_noalloc(fake, fake, fake, fake, fake, C.byref(kv), fake, fake, fake, 200, 33, 28,
+                                      0.088, fake, None) == 2
+    # a shape that fits passes the check and only then needs the device
+    assert lib.cure_tree_attn_workspace_size(4, 33, 28, C.byref(kv)) <= scratch
+    assert lib.cure_tree_attn_noalloc(fake, fake, fake, fake, fake, C.byref(kv), fake, fake, fake, 4, 33, 28,
+                                      0.088, fake, None) == 3
+
+
+def test_sampling_temperature_must_give_a_finite_scale(lib):
+    """log2(e) / T must be a finite float32: subnormal temperatures are
+    rejected before anything launches."""
+    null = C.c_void_p(0)
+    for bad in (0.0, -1.0, float("inf"), float("nan"), 1e-45, 4e-39):
+        assert lib.cure_sample_target(null, null, bad, 1, 4, 10, null, null, null) == 1, bad
+    # zero sequences with a valid temperature is a no-op
+    assert lib.cure_sample_target(null, null, 5e-39, 0, 4, 10, null, null, null) == 0
+
+
+def test_lm_head_host_checks(lib):
+    """Shapes the fused LM head cannot take are refused before any launch."""
+    null = C.c_void_p(0)
+    fake = C.c_void_p(1 << 20)
+    # negative rows, d_model below one K slice, empty vocabulary
+    assert lib.cure_lm_head_argmax(null, null, -1, 128, 10, null, null, null, 0, null) == 1
+    assert lib.cure_lm_head_argmax(null, null, 4, 32, 10, null, null, null, 0, null) == 1
+    assert lib.cure_lm_head_argmax(null, null, 4, 128, 0, null, null, null, 0, null) == 1
+    # d_model not a multiple of 64
+    assert lib.cure_lm_head_argmax(null, null, 4, 96, 10, null, null, null, 0, null) == 5
+    # zero rows is a no-op; missing pointers are rejected
+    assert lib.cure_lm_head_argmax(null, null, 0, 128, 10, null, null, null, 0, null) == 0
+    assert lib.cure_lm_head_argmax(fake, null, 4, 128, 10, null, fake, fake, 1 << 20, null) == 1
+    # misaligned hidden state
+    assert lib.cure_lm_head_argmax(C.c_void_p((1 << 20) + 2), fake, 4, 128, 10, null, fake, fake, 1 << 20,
+                                   null) == 1
+    assert lib.cure_lm_head_workspace_size(-1, 10) == 0
+    assert lib.cure_lm_head_workspace_size(4, 0) == 0
+    n = lib.cure_lm_head_workspace_size(817, 151936)
+    assert n >= 817 * 8 and n % 256 == 0
+    # a workspace smaller than the plan's is refused
+    assert lib.cure_lm_head_argmax(fake, fake, 817, 4096, 151936, null, fake, fake, n - 256, null) == 2

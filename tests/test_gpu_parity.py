@@ -82,6 +82,29 @@ def test_score_draft_full_serve_shape_sampled(cure):
     _check_scores(cure, d.logits, w.topk, rows)
 
 
+@pytest.mark.parametrize("rows,V,k", [(1024, 151936, 3), (960, 32003, 4), (912, 50021, 6), (1000, 4099, 8)])
+def test_score_draft_one_cta_per_row(cure, rows, V, k):
+    """Row counts that give every SM six CTAs take the one-CTA-per-row launch
+    (no cluster merge); the top-k, margin and log-probability epilogue of that
+    launch on sampled rows, half of them with many exact ties and -inf."""
+    rng = np.random.default_rng(rows + V + k)
+    x = rng.standard_normal((rows, V), dtype=np.float32)
+    tied = rng.random(rows) < 0.5
+    x[tied] = np.round(x[tied] * 2.0) * 0.5
+    x[tied, : V // 7] = -np.inf
+    sel = np.concatenate([np.arange(4), rng.choice(rows, size=60, replace=False)])
+    _check_scores(cure, W.to_bf16(x), k, sel)
+
+
+def test_score_draft_full_long_shape_sampled(cure):
+    """batch 64 x block 16 x vocab 128256 with top-2: 1024 rows, one CTA per
+    row, the launch the long-context configuration takes; 64 sampled rows."""
+    w = W.WORKLOADS["long64"]
+    d = W.draft_block(w)
+    rows = np.random.default_rng(1).choice(w.batch * w.block, size=64, replace=False)
+    _check_scores(cure, d.logits, w.topk, rows)
+
+
 def _tree_inputs(w, seed=None):
     d = W.draft_block(w, seed=seed)
     x = _f64(d.logits).reshape(-1, w.vocab)
@@ -550,6 +573,67 @@ def test_accept_workloads(cure, name):
         assert np.array_equal(acc[key].cpu().numpy(), o_acc[key]), key
 
 
+def test_accept_full_long_shape_sampled(cure):
+    """The long-context shape's target argmax (64 x 49 rows of 128256 logits,
+    one CTA per row) and walk with depth-2 repairs.  The oracle recomputes 8
+    sampled sequences (the largest tree among them); every other valid row
+    must give the planted id, which lies 8 above N(0, 1) noise."""
+    w = W.WORKLOADS["long64"]
+    wt = w.replace(vocab=4096)          # the tree does not depend on V
+    d, ids, margin = _tree_inputs(wt)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, w.budget, w.branches, 2, d.redraft)
+    truth = W.target_truth(wt, d, w.seed)
+    planted = W.synthetic_target_ids(truth, t["n_nodes"], t["tok"], t["parent"], t["depth"], w.vocab, w.seed)
+    B, N, V = w.batch, w.n_max, w.vocab
+    g = torch.Generator(device=DEV).manual_seed(w.seed)
+    x = torch.randn(B, N, V, generator=g, device=DEV).to(torch.bfloat16)
+    pid = torch.from_numpy(planted).to(DEV)
+    x.scatter_(2, pid[:, :, None], 8.0)
+    acc = cure.cure_accept(_gpu_tree_dict(t), w.block, target_logits=x)
+    g_targ = acc["targ"].cpu().numpy()
+    n = t["n_nodes"]
+    for b in range(B):
+        assert np.array_equal(g_targ[b, :n[b]], planted[b, :n[b]]), b
+        assert (g_targ[b, n[b]:] == -1).all()
+    rng = np.random.default_rng(2)
+    S = np.unique(np.concatenate([[int(np.argmax(n))], rng.choice(B, size=7, replace=False)]))
+    o_targ = np.full((len(S), N), -1, dtype=np.int64)
+    for i, b in enumerate(S):
+        o_targ[i, :n[b]] = oracle.row_argmax(_f64(x[b, :n[b]]))
+        assert np.array_equal(g_targ[b, :n[b]], o_targ[i, :n[b]]), b
+    o_acc = oracle.accept(o_targ, n[S], t["tok"][S], t["parent"][S], t["depth"][S], t["anc"][S], w.block)
+    for key in ("accept_len", "best_node", "path_nodes", "out_tokens", "diverge_depth"):
+        assert np.array_equal(acc[key].cpu().numpy()[S], o_acc[key]), key
+    assert cure.cure_device_error() == 0
+
+
+@pytest.mark.parametrize("name", ["sweep16", "serve32", "single8b"])
+def test_budget_zero_is_prefix_verification_on_the_gpu(cure, name):
+    """R = 0 (Sec. 3.1, Eq. 1 with no repair nodes): the tree is the draft
+    chain alone, and the walk must accept exactly the longest prefix of the
+    chain that the target's tokens confirm, i.e. plain block-parallel prefix
+    verification, computed here by a direct scan."""
+    w = W.WORKLOADS[name].replace(vocab=4096, budget=0)
+    d, ids, margin = _tree_inputs(w)
+    L = W.cache_lengths(w)
+    t = oracle.build_tree(ids, margin, d.root_tok, L, w.tau, 0, w.branches, 1)
+    assert (t["n_nodes"] == w.block + 1).all()
+    truth = W.target_truth(w, d, w.seed)
+    targ = W.synthetic_target_ids(truth, t["n_nodes"], t["tok"], t["parent"], t["depth"], w.vocab, w.seed)
+    acc = cure.cure_accept(_gpu_tree_dict(t), w.block, targ=torch.from_numpy(targ.astype(np.int32)).to(DEV))
+    a = acc["accept_len"].cpu().numpy()
+    dv = acc["diverge_depth"].cpu().numpy()
+    out = acc["out_tokens"].cpu().numpy()
+    for b in range(w.batch):
+        e = 0
+        while e < w.block and t["tok"][b, e + 1] == targ[b, e]:
+            e += 1
+        assert a[b] == e, (b, a[b], e)
+        assert dv[b] == -1
+        assert list(out[b, :e + 1]) == list(t["tok"][b, 1:e + 1]) + [targ[b, e]]
+
+
 @pytest.mark.parametrize("seed", range(8))
 def test_accept_random_trees_with_ids(cure, seed):
     """Random trees (depth-2 repairs included) with small-alphabet targets so
@@ -571,9 +655,23 @@ def test_accept_random_trees_with_ids(cure, seed):
 
 
 # ------------------------------------------------------ stochastic verification
-def _valid_sample(x, T, u, y, tol=1e-4):
+def _sum_tol(V):
+    """Relative bound on the kernel's float32 cumulative sums for a row of V
+    ids: each lane adds 8 * ceil(V / 1024) terms in sequence (four warp
+    segments of 32 lanes, eight ids per group), the walk adds up to
+    ceil(V / 1024) chunk totals, and the warp and segment reductions, the
+    rescales and the chunk scan add fewer than 64 more roundings; each
+    rounding contributes at most 2^-24 of the sum, and ex2.approx a further
+    2^-20 (its relative error, with room)."""
+    c = -(-V // 1024)
+    return (9 * c + 64) * 2.0 ** -24 + 2.0 ** -20
+
+
+def _valid_sample(x, T, u, y, tol=None):
     """y is a valid inverse-CDF draw for u: an id of nonzero probability whose
-    cumulative range (float64) contains u Z, up to float32 summation (tol Z)."""
+    cumulative range (float64) contains u Z, up to the kernel's float32
+    summation bound (tol Z)."""
+    tol = _sum_tol(len(x)) if tol is None else tol
     m = x.max()
     if m == -np.inf:
         return y == 0
@@ -612,6 +710,33 @@ def test_sample_target_inverse_cdf(cure, V, T):
             else:
                 assert _valid_sample(xf[b, j], T, float(u[b, j]), int(got[b, j])), (b, j, got[b, j])
     assert got[2, 1] == 17 and got[2, 2] == 0 and got[3, 0] >= V // 2
+
+
+@pytest.mark.parametrize("T", [1e-30, 1e-38])
+def test_sample_target_tiny_temperature_and_huge_logits(cure, T):
+    """Temperatures so small that every logit below the maximum has
+    probability 0 pick among the ids holding the maximum by the uniform (the
+    T -> 0 limit), and logits near the bf16 limit do not overflow: the draws
+    equal the oracle's exact inverse CDF (no u near a step boundary)."""
+    rng = np.random.default_rng(7)
+    B, N, V = 3, 6, 5000
+    x = rng.standard_normal((B, N, V)).astype(np.float32)
+    ties = rng.choice(V, size=3, replace=False)
+    x[0, :, ties] = 9.0                               # three ids share the maximum
+    x[1, :, :] = rng.uniform(-3e38, 1e38, size=(N, V)).astype(np.float32)
+    x[1, :, 4321] = 3.0e38                            # a maximum near the bf16 limit
+    x[2, :, :] = -np.inf
+    x[2, :, [5, 17]] = -3.0e38                        # the maximum is very negative
+    logits = W.to_bf16(x)
+    u = np.tile(np.array([0.05, 0.2, 0.4, 0.6, 0.8, 0.95], np.float32), (B, 1))
+    n = np.full(B, N, dtype=np.int32)
+    got = cure.cure_sample_target(logits.to(DEV), torch.from_numpy(n).to(DEV), torch.from_numpy(u).to(DEV),
+                                  T).cpu().numpy()
+    assert cure.cure_device_error() == 0
+    want = oracle.sample_target(_f64(logits), n, u.astype(np.float64), T)
+    assert np.array_equal(got, want)
+    assert set(got[0].tolist()) == set(ties.tolist()) and (got[1] == 4321).all()
+    assert set(got[2].tolist()) <= {5, 17}
 
 
 def test_sample_target_frequencies_follow_softmax(cure):
