@@ -501,6 +501,51 @@ def sweep_points(wl, dev, steps, warmup, world, rank):
     return out
 
 
+def profile_stage(args):
+    """Runs one stage alone on the configuration's shapes, `--steps` calls
+    after `--warmup`, and prints nothing: the command an ncu capture of that
+    stage's kernel wraps (a few GB on the device at most)."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_00531_gb300 import cure, workload as W
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = W.WORKLOADS[args.workload]
+    g = torch.Generator(device=dev).manual_seed(7)
+    name = args.profile_stage
+    if name == "lm_head":
+        rows = int(round(w.batch * (w.block + 1 + 0.55 * w.budget)))   # about the realised tree nodes
+        d_model = D_MODEL[w.name]
+        wl = (torch.randn(w.vocab, d_model, generator=g, device=dev) * d_model ** -0.5).to(torch.bfloat16)
+        h = torch.randn(rows, d_model, generator=g, device=dev).to(torch.bfloat16)
+        out = torch.empty(rows, dtype=torch.int32, device=dev)
+        ws = torch.empty(max(256, cure.cure_lm_head_workspace_size(rows, w.vocab)), dtype=torch.uint8, device=dev)
+        fn = lambda: cure.cure_lm_head_argmax(h, wl, out=out, workspace=ws)  # noqa: E731
+    elif name in ("sample", "argmax"):
+        B, N = w.batch, w.n_max
+        tl = torch.randn(B, N, w.vocab, generator=g, device=dev).to(torch.bfloat16)
+        n = torch.full((B,), N, dtype=torch.int32, device=dev)
+        uni = torch.rand(B, N, generator=g, device=dev)
+        targ = torch.empty(B, N, dtype=torch.int32, device=dev)
+        if name == "sample":
+            fn = lambda: cure.cure_sample_target(tl, n, uni, 0.8, out=targ)  # noqa: E731
+        else:
+            tree = dict(n_nodes=n, tok=torch.zeros(B, N, dtype=torch.int32, device=dev),
+                        parent=torch.zeros(B, N, dtype=torch.int32, device=dev),
+                        depth=torch.zeros(B, N, dtype=torch.int32, device=dev),
+                        anc=torch.ones(B, N, (N + 63) // 64, dtype=torch.int64, device=dev))
+            fn = lambda: cure.cure_accept(tree, w.block, target_logits=tl, targ=targ)  # noqa: E731
+    elif name == "scan":
+        x = W.draft_block(w).logits.to(dev)
+        fn = lambda: cure.cure_score_draft(x, w.topk)  # noqa: E731
+    else:
+        raise SystemExit(f"unknown stage {name}")
+    for _ in range(args.warmup + args.steps):
+        fn()
+    torch.cuda.synchronize()
+    assert cure.cure_device_error() == 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -514,7 +559,12 @@ def main():
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help=argparse.SUPPRESS)
+    ap.add_argument("--profile-stage", default=None, choices=["lm_head", "sample", "argmax", "scan"],
+                    help="run one stage alone (for a profiler capture) and print nothing")
     args = ap.parse_args()
+    if args.profile_stage:
+        profile_stage(args)
+        return
     args.warmup = max(3, args.warmup)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))

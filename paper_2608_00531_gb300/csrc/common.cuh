@@ -96,9 +96,10 @@ cudaError_t launch_resync(int layers, const LayerPtrs& caches, const cure_kv_des
                           int* err, cudaStream_t s);
 
 // Fused LM head + argmax: launch plan for a shape (persistent CTAs, one
-// 128-row M tile each, vocab N tiles of 256 split into `groups` ranges).
+// 128-row M tile each, the vocabulary's 128-id halves split into `groups`
+// ranges).
 struct LmPlan {
-  int m_tiles = 0, n_tiles = 0, groups = 0;
+  int m_tiles = 0, h_tiles = 0, groups = 0;
   size_t ws_bytes = 0;  // per-range (max, id) partials: groups * rows * 8 bytes
 };
 LmPlan plan_lm_head(int rows, int vocab);

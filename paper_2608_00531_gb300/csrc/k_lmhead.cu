@@ -5,9 +5,11 @@
 // so that the rows x vocab logits never reach HBM.
 //
 // The contraction runs on the tcgen05 tensor cores: one persistent CTA per SM
-// owns one 128-row M tile of `hidden` and a contiguous range of 256-id vocab
-// (N) tiles; the CTAs that share an N range run side by side, so each weight
-// tile is read from HBM about once and served to the other M tiles from L2.
+// owns one 128-row M tile of `hidden` and a contiguous range of the vocabulary
+// in 128-id halves, taken as 256-id (N) tiles and, for an odd count, one
+// 128-id tile at its end; the CTAs that share a vocab range run side by side,
+// so each weight tile is read from HBM about once and served to the other M
+// tiles from L2.
 //   warp 0   producer: TMA loads of the 64-wide K slices of the hidden tile
 //            [128 x 64] and of the weight tile [256 x 64] (128-byte swizzle)
 //            into a 4-stage ring;
@@ -56,7 +58,7 @@ constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
 struct LmArgs {
   int M, d, V;
-  int m_tiles, groups, n_tiles;
+  int m_tiles, groups, h_tiles;  // M tiles, vocab ranges, 128-id vocab halves
   float* part_val;   // [groups][M]
   int32_t* part_idx; // [groups][M]
   int* err;
@@ -117,9 +119,10 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
 
   const int m_tile = blockIdx.x % A.m_tiles;
   const int g = blockIdx.x / A.m_tiles;
-  const int n_lo = (int)((int64_t)g * A.n_tiles / A.groups);
-  const int n_hi = (int)((int64_t)(g + 1) * A.n_tiles / A.groups);
-  const int ntl = n_hi - n_lo;
+  const int h_lo = (int)((int64_t)g * A.h_tiles / A.groups);
+  const int h_hi = (int)((int64_t)(g + 1) * A.h_tiles / A.groups);
+  const int ntl = (h_hi - h_lo + 1) / 2;  // N tiles: 256 ids, the last one 128 for an odd count
+  auto wide = [&](int t) { return h_hi - h_lo - 2 * t >= 2; };
   const int KS = A.d / BK;
 
   if (threadIdx.x == 0) {
@@ -152,7 +155,7 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
       int it = 0;
       bool ok = true;
       for (int t = 0; t < ntl && ok; ++t) {
-        const int n = n_lo + t;
+        const int v0 = (h_lo + 2 * t) * 128;
         for (int k = 0; k < KS; ++k, ++it) {
           const int s = it % NS;
           if (it >= NS && !wait_bounded(bar(B_EMPTY + s), ((it / NS) & 1) ^ 1, abort_flag, A.err, true)) {
@@ -162,7 +165,8 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
           mbar_arrive_expect_tx(bar(B_FULL + s), kStage);
           const uint32_t st = sb + s * kStage;
           tma_load_2d(st, &mh, bar(B_FULL + s), k * BK, m_tile * BM);
-          tma_load_2d(st + kABytes, &mw, bar(B_FULL + s), k * BK, n * BN);
+          // a 128-id tile still loads a whole box; its second half goes unused
+          tma_load_2d(st + kABytes, &mw, bar(B_FULL + s), k * BK, v0);
         }
       }
       if (!ok) {  // let the copies in flight land before the CTA's smem goes away
@@ -173,7 +177,8 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false);
+      constexpr uint32_t idesc_w = idesc_bf16_f32(BM, BN, false);
+      constexpr uint32_t idesc_h = idesc_bf16_f32(BM, BN / 2, false);
       int it = 0;
       bool ok = true;
       for (int t = 0; t < ntl && ok; ++t) {
@@ -183,6 +188,7 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
           break;
         }
         tc_fence_after();
+        const uint32_t idesc = wide(t) ? idesc_w : idesc_h;
         for (int k = 0; k < KS; ++k, ++it) {
           const int s = it % NS;
           if (!wait_bounded(bar(B_FULL + s), (it / NS) & 1, abort_flag, A.err, true)) {
@@ -212,9 +218,10 @@ lm_head_argmax_kernel(const __grid_constant__ CUtensorMap mh, const __grid_const
       const bool ok = wait_bounded(bar(B_ACCFULL + a), (t >> 1) & 1, abort_flag, A.err, true);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
-      const int v0 = (n_lo + t) * BN;
+      const int v0 = (h_lo + 2 * t) * 128;
+      const int nc = wide(t) ? BN / 32 : BN / 64;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = 0; c < nc; ++c) {
         uint32_t r[32];
         tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + a * BN + c * 32, r);
         tmem_wait_ld();
@@ -309,11 +316,11 @@ bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows, int d, int b
 LmPlan plan_lm_head(int rows, int vocab) {
   LmPlan p;
   p.m_tiles = (rows + BM - 1) / BM;
-  p.n_tiles = (vocab + BN - 1) / BN;
+  p.h_tiles = (vocab + 127) / 128;
   const int sms = num_sms();
   int groups = sms / (p.m_tiles > 0 ? p.m_tiles : 1);
   if (groups < 1) groups = 1;
-  if (groups > p.n_tiles) groups = p.n_tiles;
+  if (groups > p.h_tiles) groups = p.h_tiles;
   p.groups = groups;
   p.ws_bytes = ((size_t)groups * rows * (sizeof(float) + sizeof(int32_t)) + 255) / 256 * 256;
   return p;
@@ -342,7 +349,7 @@ cudaError_t launch_lm_head_argmax(const LmPlan& p, const uint16_t* hidden, const
   a.V = vocab;
   a.m_tiles = p.m_tiles;
   a.groups = p.groups;
-  a.n_tiles = p.n_tiles;
+  a.h_tiles = p.h_tiles;
   a.part_val = static_cast<float*>(workspace);
   a.part_idx = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) + (size_t)p.groups * rows * sizeof(float));
   a.err = err;
