@@ -28,6 +28,8 @@
 // every id below the maximum gets mass 0 and the draw picks among the maxima.
 #include <float.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace cure {
@@ -80,6 +82,49 @@ struct RowView {
   }
 };
 
+// Pairs of floats in one 64-bit register pair, for the packed f32x2
+// arithmetic of sm_100 and later (two lanes of work per instruction).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float max3s(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// The (lo, hi) logit pair of one 32-bit word of a group.
+__device__ __forceinline__ uint64_t pair_of(uint32_t w) {
+  return f2_pack(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
+// The largest of a group's eight logits.
+__device__ __forceinline__ float group_max_raw(const uint4& r) {
+  const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+  float v[8];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    v[2 * q] = __uint_as_float(w[q] << 16);
+    v[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
+  }
+  return max3s(max3s(v[0], v[1], v[2]), max3s(v[3], v[4], v[5]), fmaxf(v[6], v[7]));
+}
+
 __device__ __forceinline__ void unpack8(const uint4& r, float x[8]) {
   const uint32_t w[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
@@ -99,10 +144,6 @@ __device__ __forceinline__ float warp_sum_s(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
-}
-
-__device__ __forceinline__ float group_max(const float x[8]) {
-  return fmaxf(fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])), fmaxf(fmaxf(x[4], x[5]), fmaxf(x[6], x[7])));
 }
 
 // Mass of one group against `base` (a finite logit value).
@@ -149,40 +190,64 @@ sample_target_kernel(const uint16_t* __restrict__ logits, const float* __restric
   float base = -INFINITY;  // warp-uniform
   float bm = 0.f;          // current block's mass (warp-uniform)
   int blk = 0, in_blk = 0;
+  uint64_t acc2 = f2_pack(0.f, 0.f);  // this lane's part of the current step's mass, as a pair
+  // interior groups need no per-element bounds: [gf_lo, gf_hi) lie wholly inside the row
+  const int gf_lo = rv.mis == 0 ? 0 : 1;
+  const int gf_hi = (vocab + rv.mis) >> 3;
+  const uint64_t sc2 = f2_pack(scale, scale);
   uint4 r4[kSampleUnroll];
 #pragma unroll
   for (int u = 0; u < kSampleUnroll; ++u) {
     const int g = g_lo + lane + 32 * u;
     if (g < g_hi) r4[u] = rv.load(g);
   }
-  for (int g0 = g_lo; g0 < g_hi; g0 += kStepGroups) {
+  // one warp step over groups g0 .. g0 + 127; FULL: every group of every lane
+  // is whole and inside the segment, so no check is needed
+  auto step = [&](int g0, auto full_tag) {
+    constexpr bool FULL = decltype(full_tag)::value;
     uint4 nx[kSampleUnroll];
 #pragma unroll
     for (int u = 0; u < kSampleUnroll; ++u) {
       const int g = g0 + lane + 32 * (kSampleUnroll + u);
-      if (g < g_hi) nx[u] = rv.load(g);
+      if (g < g_hi) nx[u] = (g >= gf_lo && g < gf_hi) ? ld_row(rv.vbase + g) : rv.load(g);
     }
-    float x[kSampleUnroll][8];
     float gm = -INFINITY;
 #pragma unroll
-    for (int u = 0; u < kSampleUnroll; ++u) {
-      unpack8(r4[u], x[u]);
-      if (g0 + lane + 32 * u < g_hi) gm = fmaxf(gm, group_max(x[u]));
-    }
+    for (int u = 0; u < kSampleUnroll; ++u)
+      if (FULL || g0 + lane + 32 * u < g_hi) gm = fmaxf(gm, group_max_raw(r4[u]));
     // raise the base when some lane's terms would exceed 2^kRaise
     if (__any_sync(0xffffffffu, gm > base && (base == -INFINITY || (gm - base) * scale > kRaise))) {
       const float nb = warp_max_s(gm);
-      if (base != -INFINITY) bm *= ex2s((base - nb) * scale);
+      if (base != -INFINITY) {
+        const float f = ex2s((base - nb) * scale);
+        bm *= f;
+        acc2 = f2_mul(acc2, f2_pack(f, f));
+      }
       base = nb;
     }
-    float ps = 0.f;
     if (base != -INFINITY) {
+      // p = 2^((l - base) scale): a packed subtraction and product per pair;
+      // never l * scale - base * scale, whose rounding error can be huge in
+      // exponent units when scale is large
+      const uint64_t nb2 = f2_pack(-base, -base);
 #pragma unroll
-      for (int u = 0; u < kSampleUnroll; ++u)
-        if (g0 + lane + 32 * u < g_hi) ps += group_mass(x[u], base, scale);
+      for (int u = 0; u < kSampleUnroll; ++u) {
+        if (FULL || g0 + lane + 32 * u < g_hi) {
+          const uint32_t w[4] = {r4[u].x, r4[u].y, r4[u].z, r4[u].w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            float a, b;
+            f2_unpack(f2_mul(f2_add(pair_of(w[q]), nb2), sc2), a, b);
+            acc2 = f2_add(acc2, f2_pack(ex2s(a), ex2s(b)));
+          }
+        }
+      }
     }
-    bm += warp_sum_s(ps);
     if (++in_blk == bstride || g0 + kStepGroups >= g_hi) {
+      float a, b;
+      f2_unpack(acc2, a, b);
+      bm += warp_sum_s(a + b);
+      acc2 = f2_pack(0.f, 0.f);
       if (lane == 0) {
         s_blk[warp][blk] = bm;
         s_blkbase[warp][blk] = base;
@@ -193,7 +258,14 @@ sample_target_kernel(const uint16_t* __restrict__ logits, const float* __restric
     }
 #pragma unroll
     for (int u = 0; u < kSampleUnroll; ++u) r4[u] = nx[u];
-  }
+  };
+  int g0 = g_lo;
+  // a partial first group (a row not on a 16-byte boundary) is checked; then
+  // full steps while this step's groups and the next step's loads are whole
+  // and in range; then the checked tail
+  for (; g0 < g_hi && g0 < gf_lo; g0 += kStepGroups) step(g0, std::integral_constant<bool, false>());
+  for (; g0 + 2 * kStepGroups <= min(g_hi, gf_hi); g0 += kStepGroups) step(g0, std::integral_constant<bool, true>());
+  for (; g0 < g_hi; g0 += kStepGroups) step(g0, std::integral_constant<bool, false>());
   __syncwarp();
   // the segment's mass at its final base (bases only grow)
   float sm = 0.f;
