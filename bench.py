@@ -45,7 +45,7 @@ import torch  # noqa: E402
 # DRAM bytes (read + write) of one tree-attention launch on this workload, from
 # one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
 # source with the given sha256 prefix; another source reports null
-ATTN_TRAFFIC = {"2d1748d0f70bce81": 312700160}
+ATTN_TRAFFIC = {"e317c2d16bc227d7": 314443520}
 
 DEFAULT_WORKLOAD = "serve32"
 # the target model width behind each configuration's LM head (for the fused

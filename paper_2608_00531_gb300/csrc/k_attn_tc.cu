@@ -250,6 +250,13 @@ __device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
       : "memory");
 }
+// An L2 prefetch of one 4-D box (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_4d(const CUtensorMap* map, int c0, int c1, int c2, int c3) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
+}
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
                                             int c0, int c1, int c2, int c3) {
   asm volatile(
@@ -477,6 +484,16 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
       const Seg s = sch.at(g, g_end);
       g = s.next;
       if (s.t1 <= s.t0) continue;
+      // the next piece's Q boxes are prefetched into L2 now, so that its Q
+      // load at the piece boundary is served from L2
+      if (g < g_end && lane == 0) {
+        const Seg nx = sch.at(g, g_end);
+        if (nx.t1 > nx.t0) {
+          for (int m = 0; m < (active1(nx) ? 2 : 1); ++m)
+            for (int hf = 0; hf < 2; ++hf)
+              tma_prefetch_4d(&tm_q, hf * 64, 0, nx.h, nx.b * A.n_max + (2 * nx.rg + m) * npb);
+        }
+      }
       // Q of both M tiles once the previous piece's S products are done; it
       // is requested after the piece's first K/V tile, whose ring stage frees
       // up independently, so that the ring refills across the piece boundary

@@ -153,5 +153,6 @@ class RepairVerifyStep:
     @property
     def launches_per_step(self) -> int:
         """Library kernels one step launches: scan, tree, one attention kernel per
-        layer, target argmax + walk, gather + finalize."""
-        return 1 + 1 + self.layers + 2 + 2
+        layer, target argmax + walk, and the resync gather (its finalize runs in
+        the gather's grid, since the step's new lengths do not alias the old)."""
+        return 1 + 1 + self.layers + 2 + 1
