@@ -261,8 +261,8 @@ __device__ __forceinline__ void consume1(float x, int idx, TopK<KT>& tk, Lse2& l
 // leaves the loads in flight as the limit).  grid (S, rows) with cluster
 // (S, 1, 1).  TARGET: rows are (b, j) of a [batch][n_max] tree and only
 // j < n_nodes[b] are scanned.
-template <int KT, bool LSE, bool TARGET>
-__global__ void __launch_bounds__(kCtaThreads, 6)
+template <int KT, bool LSE, bool TARGET, int CW>
+__global__ void __launch_bounds__(CW * 32 + 32, CW == 4 ? 6 : 4)
 vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int n_max,
                   const int32_t* __restrict__ n_nodes, int32_t* __restrict__ top_ids,
                   float* __restrict__ top_vals, float* __restrict__ margin,
@@ -314,7 +314,7 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   if (tid == 0) {
     for (int st = 0; st < kStages; ++st) {
       bar_init(smem_addr(&full_bar[st]), 1);
-      bar_init(smem_addr(&empty_bar[st]), kWarps);
+      bar_init(smem_addr(&empty_bar[st]), CW);
     }
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -416,7 +416,7 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     }
   };
 
-  if (warp == kWarps) {
+  if (warp == CW) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
       int issued = 0;
@@ -448,14 +448,16 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       uint4 r[kUnroll];
       int gi[kUnroll];
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
+      constexpr int kSteps = kChunkVec / (CW * 32 * kUnroll);  // steps per chunk
+#pragma unroll
+      for (int half = 0; half < kSteps; ++half) {
 #pragma unroll
         for (int u = 0; u < kUnroll; ++u) {
-          const int o = warp * 32 + lane + (half * kUnroll + u) * kThreads;
+          const int o = warp * 32 + lane + (half * kUnroll + u) * (CW * 32);
           gi[u] = cb + o;
           if (full || gi[u] < lim) r[u] = ld_shared_v4(smem_addr(&ring[st][o]));
         }
-        if (half == 1) {
+        if (half == kSteps - 1) {
           __syncwarp();
           if (lane == 0) bar_arrive(smem_addr(&empty_bar[st]));  // this warp's vectors are in registers
         }
@@ -482,9 +484,9 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   }
 
   // ---- CTA merge
-  __shared__ Part<KT, LSE> warp_part[kWarps];
+  __shared__ Part<KT, LSE> warp_part[CW];
   __shared__ Part<KT, LSE> cta_part;
-  if (lane == 0 && warp < kWarps) {
+  if (lane == 0 && warp < CW) {
 #pragma unroll
     for (int k = 0; k < KT; ++k) {
       warp_part[warp].v[k] = tk.v[k];
@@ -498,7 +500,7 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     tk.init();
     ls.mb = -INFINITY;
     ls.s = 0.f;
-    if (lane < kWarps) {
+    if (lane < CW) {
 #pragma unroll
       for (int k = 0; k < KT; ++k) {
         tk.v[k] = warp_part[lane].v[k];
@@ -508,7 +510,7 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       ls.s = warp_part[lane].s;
     }
 #pragma unroll
-    for (int off = kWarps / 2; off > 0; off >>= 1) {
+    for (int off = CW / 2; off > 0; off >>= 1) {
       tk.merge_shfl(off);
       if constexpr (LSE) {
         const float mb2 = __shfl_xor_sync(0xffffffffu, ls.mb, off);
@@ -846,9 +848,9 @@ int pick_split_lsu(int64_t rows, int vocab) {
 #ifndef CURE_SCAN_SPLIT_CEIL
 #define CURE_SCAN_SPLIT_CEIL 0
 #endif
-int pick_split_ring(int64_t rows, int vocab) {
+int pick_split_ring(int64_t rows, int vocab, int per_sm) {
   const int nvec = vocab / 8;
-  const int64_t slots = 6LL * num_sms();
+  const int64_t slots = (int64_t)per_sm * num_sms();
   if (rows >= slots) return 1;
   int s = (int)(CURE_SCAN_SPLIT_CEIL ? (slots + rows - 1) / rows : slots / rows);
   s = max(1, min(s, 8));
@@ -856,14 +858,14 @@ int pick_split_ring(int64_t rows, int vocab) {
   return s;
 }
 
-template <int KT, bool LSE, bool TARGET, bool RING>
+template <int KT, bool LSE, bool TARGET, bool RING, int CW = 4>
 cudaError_t launch_scan(const uint16_t* logits, int64_t rows, int vocab, int k_out, int n_max,
                         const int32_t* n_nodes, int32_t* top_ids, float* top_vals, float* margin,
                         float* logp1, cudaStream_t s) {
-  const int S = RING ? pick_split_ring(rows, vocab) : pick_split_lsu(rows, vocab);
+  const int S = RING ? pick_split_ring(rows, vocab, CW == 4 ? 6 : 4) : pick_split_lsu(rows, vocab);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, (unsigned)rows, 1);
-  cfg.blockDim = dim3(RING ? kCtaThreads : kThreads, 1, 1);
+  cfg.blockDim = dim3(RING ? CW * 32 + 32 : kThreads, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
@@ -876,7 +878,7 @@ cudaError_t launch_scan(const uint16_t* logits, int64_t rows, int vocab, int k_o
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   if constexpr (RING)
-    return cudaLaunchKernelEx(&cfg, vocab_ring_kernel<KT, LSE, TARGET>, logits, vocab, k_out, n_max, n_nodes,
+    return cudaLaunchKernelEx(&cfg, vocab_ring_kernel<KT, LSE, TARGET, CW>, logits, vocab, k_out, n_max, n_nodes,
                               top_ids, top_vals, margin, logp1, device_error_word());
   else
     return cudaLaunchKernelEx(&cfg, vocab_scan_kernel<KT, LSE, TARGET>, logits, vocab, k_out, n_max, n_nodes,
