@@ -83,6 +83,20 @@ def test_lm_head_argmax_small_shapes(cure, rows, d, V):
     assert exact >= 0.8 * rows
 
 
+def test_lm_head_argmax_more_m_tiles_than_sms(cure):
+    """More 128-row tiles than SMs: one vocab range per tile and a grid of
+    more than one wave."""
+    rng = np.random.default_rng(8)
+    rows, d, V = 160 * 128 + 37, 64, 700
+    h = W.to_bf16(rng.standard_normal((rows, d)).astype(np.float32))
+    w = W.to_bf16((rng.standard_normal((V, d)) / np.sqrt(d)).astype(np.float32))
+    got = cure.cure_lm_head_argmax(h.to(DEV), w.to(DEV)).cpu().numpy()
+    assert cure.cure_device_error() == 0
+    sel = np.concatenate([np.arange(64), rows - 64 + np.arange(64), rng.choice(rows, 128, replace=False)])
+    exact = _check(got[sel], W.bf16_to_f64(h)[sel], W.bf16_to_f64(w), d)
+    assert exact >= 0.8 * len(sel)
+
+
 def test_lm_head_argmax_ties_take_the_lowest_id(cure):
     """Identical weight rows give bit-identical logits; the lowest id must win
     within a tile, across N tiles and across the CTAs' vocab ranges."""

@@ -608,6 +608,37 @@ def test_accept_full_long_shape_sampled(cure):
     assert cure.cure_device_error() == 0
 
 
+@pytest.mark.parametrize("B,N,V", [(3, 9, 4099), (2, 5, 1001), (1, 4, 8), (2, 3, 9), (4, 33, 151937),
+                                   (40, 33, 32003)])
+def test_target_argmax_ragged_rows_and_ties(cure, B, N, V):
+    """The ring-fed target argmax on rows that start off a 16-byte boundary
+    (odd vocabularies), vocabularies smaller than one vector, few rows (rows
+    split over a cluster) and many, with exact ties and -inf: the ids must be
+    the oracle's first maximum, and rows past n_nodes -1."""
+    rng = np.random.default_rng(B * 1000 + V)
+    x = (rng.integers(-4, 5, size=(B, N, V)) * 0.5).astype(np.float32)   # many exact ties
+    x[0, 0, :] = -np.inf
+    x[0, 0, V - 1] = 1.0                              # the maximum in the last id
+    if N > 1:
+        x[0, 1, :] = -np.inf                          # no finite logit: id 0
+    logits = W.to_bf16(x)
+    n = rng.integers(1, N + 1, size=B).astype(np.int32)
+    n[0] = N
+    tree = {"n_nodes": torch.from_numpy(n).to(DEV),
+            "tok": torch.zeros(B, N, dtype=torch.int32, device=DEV),
+            "parent": torch.zeros(B, N, dtype=torch.int32, device=DEV),
+            "depth": torch.zeros(B, N, dtype=torch.int32, device=DEV),
+            "anc": torch.ones(B, N, (N + 63) // 64, dtype=torch.int64, device=DEV)}
+    tree["parent"][:, 0] = -1
+    acc = cure.cure_accept(tree, 1 if N < 3 else 2, target_logits=logits.to(DEV))
+    got = acc["targ"].cpu().numpy()
+    want = oracle.row_argmax(_f64(logits).reshape(-1, V)).reshape(B, N)
+    for b in range(B):
+        assert np.array_equal(got[b, :n[b]], want[b, :n[b]]), b
+        assert (got[b, n[b]:] == -1).all()
+    assert got[0, 0] == V - 1
+
+
 @pytest.mark.parametrize("name", ["sweep16", "serve32", "single8b"])
 def test_budget_zero_is_prefix_verification_on_the_gpu(cure, name):
     """R = 0 (Sec. 3.1, Eq. 1 with no repair nodes): the tree is the draft
