@@ -327,6 +327,16 @@ cure_status cure_resync_kv(int32_t layers, void* const* k_caches, void* const* v
  * Returns CURE_ERR_DEVICE_FAULT when any bit was set, CURE_OK otherwise. */
 cure_status cure_device_error(void* stream, int32_t* bits);
 
+/*
+ * Failure-detection self-test (no counterpart in the paper): runs the
+ * library's bounded pipeline wait, the one every kernel's barrier waits go
+ * through, on a barrier that nothing ever completes, with a limit of
+ * `limit_cycles` SM clock cycles (1 .. 2^30, the kernels' own limit).  The
+ * wait gives up, raises CURE_DEVERR_TIMEOUT in the device error word and
+ * returns; cure_device_error() then reports it, and the context stays usable.
+ */
+cure_status cure_selftest_wait_timeout(int64_t limit_cycles, void* stream);
+
 /* Static description of a status code. */
 const char* cure_status_string(cure_status s);
 

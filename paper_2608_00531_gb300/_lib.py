@@ -15,11 +15,11 @@ CURE_OK = 0
 STATUS = {0: "CURE_OK", 1: "CURE_ERR_INVALID_ARG", 2: "CURE_ERR_CAPACITY", 3: "CURE_ERR_CUDA",
           4: "CURE_ERR_DEVICE_FAULT", 5: "CURE_ERR_UNSUPPORTED"}
 
-DEVERR_PAGE, DEVERR_SLOT, DEVERR_NODES, DEVERR_TOKEN = 0x1, 0x2, 0x4, 0x8
+DEVERR_PAGE, DEVERR_SLOT, DEVERR_NODES, DEVERR_TOKEN, DEVERR_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
 
 # every entry point the header declares
 EXPORTS = ("cure_score_draft", "cure_build_tree", "cure_tree_attn", "cure_tree_attn_workspace_size",
-           "cure_accept", "cure_lm_head_argmax", "cure_lm_head_workspace_size", "cure_sample_target", "cure_resync_kv", "cure_device_error", "cure_status_string",
+           "cure_accept", "cure_lm_head_argmax", "cure_lm_head_workspace_size", "cure_selftest_wait_timeout", "cure_sample_target", "cure_resync_kv", "cure_device_error", "cure_status_string",
            "cure_abi_version")
 
 
@@ -69,6 +69,8 @@ def load() -> C.CDLL:
     lib.cure_lm_head_argmax.argtypes = [P, P, I32, I32, I32, P, P, P, C.c_size_t, P]
     lib.cure_lm_head_workspace_size.argtypes = [I32, I32]
     lib.cure_lm_head_workspace_size.restype = C.c_size_t
+    lib.cure_selftest_wait_timeout.argtypes = [C.c_int64, P]
+    lib.cure_selftest_wait_timeout.restype = C.c_int
     lib.cure_resync_kv.argtypes = [I32, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
                                    C.POINTER(KVDesc), P, P, I32, I32, I32, P, P, P, P, P, P, P,
                                    P, P, P]

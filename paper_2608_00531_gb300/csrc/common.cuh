@@ -12,6 +12,13 @@ constexpr int kMaxNodes = 256;     // n_max limit: 4 ancestor words
 constexpr int kMaxLayers = 128;    // resync: layers passed by value
 constexpr int kAttnBatchLimit = 256;  // tree attention: sequences per call
 
+// An NVTX range named after the entry point, for the duration of the host
+// call (header-only NVTX: a no-op unless a profiler's tool is attached).
+struct ApiRange {
+  explicit ApiRange(const char* name);
+  ~ApiRange();
+};
+
 // Device error word of the current device (see cure_device_error).
 int* device_error_word();
 int num_sms();

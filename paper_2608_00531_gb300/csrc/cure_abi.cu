@@ -2,6 +2,8 @@
 // Nothing here allocates device memory.
 #include <cuda.h>
 #include <float.h>
+#include <nvtx3/nvToolsExt.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -112,6 +114,9 @@ cudaError_t device_symbol_address(SymbolCache* cache, const void* symbol, void**
   return cudaSuccess;
 }
 
+ApiRange::ApiRange(const char* name) { nvtxRangePushA(name); }
+ApiRange::~ApiRange() { nvtxRangePop(); }
+
 int* device_error_word() {
   static SymbolCache* cache = new_symbol_cache();
   void* p = nullptr;
@@ -154,6 +159,7 @@ const char* cure_status_string(cure_status s) {
 cure_status cure_score_draft(const void* logits, int32_t rows, int32_t vocab, int32_t topk,
                              int32_t* top_ids, float* top_vals, float* margin, float* logp1,
                              void* stream) {
+  ApiRange range("cure_score_draft");
   if (rows < 0 || vocab < 2 || topk < 2 || topk > 8 || topk > vocab) return CURE_ERR_INVALID_ARG;
   if (rows > 65535) return CURE_ERR_UNSUPPORTED;
   if (rows == 0) return CURE_OK;
@@ -167,6 +173,7 @@ cure_status cure_build_tree(const cure_tree_params* p, const int32_t* top_ids, c
                             int32_t* n_nodes, int32_t* tok, int32_t* pos, int32_t* parent,
                             int32_t* depth, uint64_t* anc, int32_t* ufp_pos, int32_t* n_ufp,
                             void* stream) {
+  ApiRange range("cure_build_tree");
   if (!p) return CURE_ERR_INVALID_ARG;
   if (p->batch < 0 || p->block < 1 || p->block > 32 || p->topk < 2 || p->topk > 8 ||
       p->budget < 0 || p->branches < 1 || p->branches > p->topk ||
@@ -200,6 +207,7 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
                            const int32_t* cache_len, const int32_t* n_nodes, const uint64_t* anc,
                            int32_t batch, int32_t n_max, int32_t heads_q, float scale, void* out,
                            void* workspace, size_t workspace_bytes, void* stream) {
+  ApiRange range("cure_tree_attn");
   cure_status why;
   if (!kv_ok(kv, &why)) return why;
   if (batch < 0 || n_max < 1 || heads_q < 1 || heads_q % kv->heads_kv != 0 ||
@@ -231,6 +239,7 @@ cure_status cure_tree_attn(const void* q, const void* tree_k, const void* tree_v
 cure_status cure_sample_target(const void* target_logits, const float* uniforms, float temperature,
                                int32_t batch, int32_t n_max, int32_t vocab, const int32_t* n_nodes,
                                int32_t* targ, void* stream) {
+  ApiRange range("cure_sample_target");
   // log2(e) / T must be a finite float: T from about 4.2e-39 up
   if (batch < 0 || n_max < 1 || vocab < 1 || !(temperature > 0.f && temperature <= FLT_MAX) ||
       !(1.4426950408889634f / temperature <= FLT_MAX))
@@ -254,6 +263,7 @@ size_t cure_lm_head_workspace_size(int32_t rows, int32_t vocab) {
 cure_status cure_lm_head_argmax(const void* hidden, const void* w_lm, int32_t rows, int32_t d_model,
                                 int32_t vocab, const int32_t* out_index, int32_t* targ, void* workspace,
                                 size_t workspace_bytes, void* stream) {
+  ApiRange range("cure_lm_head_argmax");
   if (rows < 0 || d_model < 64 || vocab < 1) return CURE_ERR_INVALID_ARG;
   if (d_model % 64 != 0) return CURE_ERR_UNSUPPORTED;
   if (rows == 0) return CURE_OK;
@@ -273,6 +283,7 @@ cure_status cure_accept(const void* target_logits, int32_t* targ, int32_t batch,
                         const int32_t* parent, const int32_t* depth, const uint64_t* anc,
                         int32_t* accept_len, int32_t* best_node, int32_t* path_nodes,
                         int32_t* out_tokens, int32_t* diverge_depth, void* stream) {
+  ApiRange range("cure_accept");
   if (batch < 0 || n_max < 1 || block < 1 || block > 32 || n_max < block + 1)
     return CURE_ERR_INVALID_ARG;
   if (n_max > kMaxNodes) return CURE_ERR_UNSUPPORTED;
@@ -301,6 +312,7 @@ cure_status cure_resync_kv(int32_t layers, void* const* k_caches, void* const* v
                            const int32_t* out_tokens, const int32_t* cache_len_in,
                            int32_t* cache_len_out, int32_t* draft_valid_len,
                            int32_t* replay_tokens, int32_t* n_replay, void* stream) {
+  ApiRange range("cure_resync_kv");
   cure_status why;
   if (!kv_ok(kv, &why)) return why;
   if (layers < 0 || layers > kMaxLayers || batch < 0 || n_max < 1 || block < 1 || block > 32 ||

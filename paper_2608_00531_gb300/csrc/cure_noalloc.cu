@@ -35,6 +35,7 @@ extern "C" cure_status cure_tree_attn_noalloc(const void* q, const void* tree_k,
                                               const int32_t* n_nodes, const uint64_t* anc,
                                               int32_t batch, int32_t n_max, int32_t heads_q,
                                               float scale, void* out, void* stream) {
+  ApiRange range("cure_tree_attn_noalloc");
   if (!kv) return CURE_ERR_INVALID_ARG;
   if (kv->layout != 0 && kv->layout != 1) return CURE_ERR_INVALID_ARG;
   if (kv->heads_kv < 1 || kv->max_len < 0) return CURE_ERR_INVALID_ARG;

@@ -96,7 +96,6 @@ static_assert(kSmemBytes <= 232448, "fits the 227 KiB opt-in");
 constexpr uint32_t kColS = 0;    // S[m]:      columns m*64
 constexpr uint32_t kColP = 128;  // P[m][buf]: columns 128 + m*64 + buf*32
 constexpr uint32_t kColO = 256;  // O[m]:      columns 256 + m*128
-constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
 // One S product group, S_m = Q_m K^T over K = 128 (8 MMAs), in one asm
 // block: the descriptors step by constant adds (16-byte units: 32 bytes
@@ -147,21 +146,6 @@ struct Bar {
   uint32_t base;
   __device__ __forceinline__ uint32_t operator()(int i) const { return base + 8u * (uint32_t)i; }
 };
-
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             int* err, bool honour_abort) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (honour_abort && *abort_flag) return false;
-    if (clock64() - t0 > kTimeoutCycles) {
-      *abort_flag = 1;
-      flag(err, CURE_DEVERR_TIMEOUT);
-      return false;
-    }
-  }
-}
 
 // All lanes of the warp wait; the warp proceeds only if every lane succeeded.
 __device__ __forceinline__ bool wait_warp(uint32_t bar, uint32_t parity, volatile int* abort_flag,

@@ -54,7 +54,6 @@ constexpr int kOffAbort = kOffTmemSlot + 4;
 constexpr int kSmemUsed = kOffAbort + 4;
 constexpr int kSmemBytes = kSmemUsed + 1024;  // room to align the base to 1024 bytes
 static_assert(kSmemBytes <= 232448, "fits the 227 KiB opt-in");
-constexpr long long kTimeoutCycles = 1LL << 30;  // about half a second
 
 struct LmArgs {
   int M, d, V;
@@ -63,21 +62,6 @@ struct LmArgs {
   int32_t* part_idx; // [groups][M]
   int* err;
 };
-
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* err,
-                                             bool honour_abort) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (honour_abort && *abort_flag) return false;
-    if (clock64() - t0 > kTimeoutCycles) {
-      *abort_flag = 1;
-      flag(err, CURE_DEVERR_TIMEOUT);
-      return false;
-    }
-  }
-}
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0, int c1) {
   asm volatile(

@@ -29,6 +29,7 @@
 #include <type_traits>
 
 #include "common.cuh"
+#include "tc_ptx.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -43,48 +44,10 @@ constexpr int kChunkVec = 512;             // 16-byte vectors per ring stage (8 
 constexpr int kStages = 3;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr long long kScanTimeoutCycles = 1LL << 30;  // about half a second
 
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void bar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool bar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Waits for the phase of the given parity; gives up after kScanTimeoutCycles
-// (or at once when `abort` is set), flagging CURE_DEVERR_TIMEOUT.
-__device__ __forceinline__ bool bar_wait(uint32_t bar, uint32_t parity, volatile int* abort, int* err,
-                                         bool honour_abort) {
-  if (bar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (true) {
-    if (bar_try_wait(bar, parity)) return true;
-    if (honour_abort && *abort) return false;
-    if (clock64() - t0 > kScanTimeoutCycles) {
-      *abort = 1;
-      flag(err, CURE_DEVERR_TIMEOUT);
-      return false;
-    }
-  }
-}
+using tc::smem_u32;
+using tc::wait_bounded;
+
 // One bulk copy of `bytes` (a multiple of 16) from global memory into this
 // CTA's shared memory, completing on `bar`.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -313,8 +276,8 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   const int nchunks = (nloc + kChunkVec - 1) / kChunkVec;
   if (tid == 0) {
     for (int st = 0; st < kStages; ++st) {
-      bar_init(smem_addr(&full_bar[st]), 1);
-      bar_init(smem_addr(&empty_bar[st]), CW);
+      tc::mbar_init(smem_u32(&full_bar[st]), 1);
+      tc::mbar_init(smem_u32(&empty_bar[st]), CW);
     }
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -423,22 +386,22 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       for (int ch = 0; ch < nchunks; ++ch, ++issued) {
         const int st = ch % kStages;
         if (ch >= kStages &&
-            !bar_wait(smem_addr(&empty_bar[st]), ((ch / kStages) & 1) ^ 1, abort_flag, err, true))
+            !wait_bounded(smem_u32(&empty_bar[st]), ((ch / kStages) & 1) ^ 1, abort_flag, err, true))
           break;
         const uint32_t bytes = (uint32_t)min(kChunkVec, nloc - ch * kChunkVec) * 16u;
-        bar_expect_tx(smem_addr(&full_bar[st]), bytes);
-        bulk_load(smem_addr(&ring[st][0]), vp + vb + ch * kChunkVec, bytes, smem_addr(&full_bar[st]));
+        tc::mbar_arrive_expect_tx(smem_u32(&full_bar[st]), bytes);
+        bulk_load(smem_u32(&ring[st][0]), vp + vb + ch * kChunkVec, bytes, smem_u32(&full_bar[st]));
       }
       // the copies in flight land before the CTA's shared memory goes away
       for (int ch = max(0, issued - kStages); ch < issued; ++ch)
-        bar_wait(smem_addr(&full_bar[ch % kStages]), (ch / kStages) & 1, abort_flag, err, false);
+        wait_bounded(smem_u32(&full_bar[ch % kStages]), (ch / kStages) & 1, abort_flag, err, false);
     }
   } else {
     // ---------------------------------------------------------------- consumers
     bool first = true;
     for (int ch = 0; ch < nchunks; ++ch) {
       const int st = ch % kStages;
-      const bool ok = bar_wait(smem_addr(&full_bar[st]), (ch / kStages) & 1, abort_flag, err, true);
+      const bool ok = wait_bounded(smem_u32(&full_bar[st]), (ch / kStages) & 1, abort_flag, err, true);
       if (!__all_sync(0xffffffffu, ok)) break;
       const int cb = ch * kChunkVec;              // chunk's first vector (vb-based)
       const int lim = nloc;
@@ -455,11 +418,11 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
         for (int u = 0; u < kUnroll; ++u) {
           const int o = warp * 32 + lane + (half * kUnroll + u) * (CW * 32);
           gi[u] = cb + o;
-          if (full || gi[u] < lim) r[u] = ld_shared_v4(smem_addr(&ring[st][o]));
+          if (full || gi[u] < lim) r[u] = ld_shared_v4(smem_u32(&ring[st][o]));
         }
         if (half == kSteps - 1) {
           __syncwarp();
-          if (lane == 0) bar_arrive(smem_addr(&empty_bar[st]));  // this warp's vectors are in registers
+          if (lane == 0) tc::mbar_arrive(smem_u32(&empty_bar[st]));  // this warp's vectors are in registers
         }
         if (full) step(r, gi, lim, first && half == 0, std::integral_constant<bool, true>());
         else step(r, gi, lim, first && half == 0, std::integral_constant<bool, false>());

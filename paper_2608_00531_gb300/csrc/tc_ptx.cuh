@@ -5,6 +5,8 @@
 #include <cuda.h>
 #include <stdint.h>
 
+#include "../../include/cure.h"
+
 namespace cure {
 namespace tc {
 
@@ -38,6 +40,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "r"(bar), "r"(parity)
       : "memory");
   return ok != 0;
+}
+
+// Bounded wait on the phase of the given parity.  Every pipeline wait in the
+// library goes through it: after `limit` cycles (about half a second by
+// default) it sets the CTA's abort flag, raises CURE_DEVERR_TIMEOUT in the
+// device error word and returns false, so that a logic error surfaces as an
+// error status instead of a hung GPU.  With `honour_abort` it also returns
+// false as soon as another role of the CTA has aborted.
+constexpr long long kWaitTimeoutCycles = 1LL << 30;
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* err,
+                                             bool honour_abort, long long limit = kWaitTimeoutCycles) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (honour_abort && *abort_flag) return false;
+    if (clock64() - t0 > limit) {
+      *abort_flag = 1;
+      if (err) atomicOr(err, CURE_DEVERR_TIMEOUT);
+      return false;
+    }
+  }
 }
 
 // ---------------------------------------------------------------- proxies

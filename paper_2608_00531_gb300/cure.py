@@ -276,6 +276,12 @@ def cure_device_error(stream=None) -> int:
     return int(bits.value)
 
 
+def cure_selftest_wait_timeout(limit_cycles: int = 1 << 24, stream=None) -> None:
+    """Runs the library's bounded wait on a barrier nothing completes (a
+    failure-detection self-test); read the outcome with cure_device_error()."""
+    check("cure_selftest_wait_timeout", _lib.load().cure_selftest_wait_timeout(int(limit_cycles), _stream(stream)))
+
+
 def cure_status_string(code: int) -> str:
     return _lib.load().cure_status_string(code).decode()
 

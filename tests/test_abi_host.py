@@ -209,3 +209,10 @@ def test_lm_head_host_checks(lib):
     assert n >= 817 * 8 and n % 256 == 0
     # a workspace smaller than the plan's is refused
     assert lib.cure_lm_head_argmax(fake, fake, 817, 4096, 151936, null, fake, fake, n - 256, null) == 2
+
+
+def test_selftest_limit_is_checked_on_the_host(lib):
+    """The failure-detection self-test takes a wait limit of 1 .. 2^30 cycles;
+    others are refused before any launch."""
+    for bad in (0, -5, (1 << 30) + 1):
+        assert lib.cure_selftest_wait_timeout(bad, None) == 1
