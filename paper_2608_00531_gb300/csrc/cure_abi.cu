@@ -142,7 +142,7 @@ using namespace cure;
 
 extern "C" {
 
-int32_t cure_abi_version(void) { return 104; }
+int32_t cure_abi_version(void) { return 105; }
 
 const char* cure_status_string(cure_status s) {
   switch (s) {

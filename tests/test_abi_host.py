@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert lib.cure_abi_version() == 104
+    assert lib.cure_abi_version() == 105
     assert lib.cure_status_string(0) == b"ok"
     assert lib.cure_status_string(2) == b"workspace too small"
 
