@@ -40,6 +40,12 @@ constexpr int kAttnMaxCtas = 256;   // persistent CTAs (one per SM, at most this
 #define CURE_ATTN_UNIT_COST 3
 #endif
 constexpr int kAttnUnitCost = CURE_ATTN_UNIT_COST;
+// Fewest tile positions (tiles plus unit costs) a CTA is given before the
+// grid shrinks below one CTA per SM (0: always one per SM).
+#ifndef CURE_ATTN_MIN_TILES
+#define CURE_ATTN_MIN_TILES 8
+#endif
+constexpr int kAttnMinTiles = CURE_ATTN_MIN_TILES;
 
 // The persistent tcgen05 kernel (writes `out`; merges split units itself).
 cudaError_t launch_tree_attn_tc(const AttnArgs& A, dim3 grid, cudaStream_t s);

@@ -65,7 +65,17 @@ cudaError_t launch_tree_attn(const AttnPlan& plan, const uint16_t* q, const uint
   A.ws_lse = reinterpret_cast<float*>(ws + plan.ws_cnt + plan.ws_o);
   A.out = out;
   A.err = err;
-  const int ctas = std::min(num_sms(), kAttnMaxCtas);
+  // One CTA per SM, unless the shape's work (bounded above from the cache
+  // capacity, since the lengths are on the device) gives a CTA fewer than
+  // kAttnMinTiles tile positions: a unit cut into many pieces costs a merge of
+  // that many partials, which the last piece does alone, so small problems
+  // take fewer, longer pieces.
+  const int64_t tiles_unit = (A.cap + kAttnKeys - 1) / kAttnKeys +
+                             (A.inplace ? 0 : (n_max + kAttnKeys - 1) / kAttnKeys);
+  const int64_t positions = (int64_t)plan.units_max * (tiles_unit + kAttnUnitCost);
+  int ctas = std::min(num_sms(), kAttnMaxCtas);
+  if (kAttnMinTiles > 0)
+    ctas = (int)std::max<int64_t>(1, std::min<int64_t>(ctas, positions / kAttnMinTiles));
   return launch_tree_attn_tc(A, dim3(ctas, 1, 1), s);
 }
 

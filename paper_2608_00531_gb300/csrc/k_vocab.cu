@@ -808,14 +808,11 @@ int pick_split_lsu(int64_t rows, int vocab) {
 // else rows split over a cluster of up to 8 CTAs, each keeping at least two
 // vectors per consumer thread.  Bytes in flight come from each CTA's ring, so
 // a CTA that streams a whole row keeps the SM as busy as several would.
-#ifndef CURE_SCAN_SPLIT_CEIL
-#define CURE_SCAN_SPLIT_CEIL 0
-#endif
 int pick_split_ring(int64_t rows, int vocab, int per_sm) {
   const int nvec = vocab / 8;
   const int64_t slots = (int64_t)per_sm * num_sms();
   if (rows >= slots) return 1;
-  int s = (int)(CURE_SCAN_SPLIT_CEIL ? (slots + rows - 1) / rows : slots / rows);
+  int s = (int)(slots / rows);
   s = max(1, min(s, 8));
   while (s > 1 && nvec / s < 2 * kThreads) --s;
   return s;
