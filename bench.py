@@ -44,8 +44,9 @@ import torch  # noqa: E402
 
 # DRAM bytes (read + write) of one tree-attention launch on this workload, from
 # one ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel
-# source with the given sha256 prefix; another source reports null
-ATTN_TRAFFIC = {"e317c2d16bc227d7": 314443520}
+# sources with the given sha256 prefix; other sources report null
+ATTN_SOURCES = ("k_attn_tc.cu", "k_attn.cu", "attn_common.cuh", "tc_ptx.cuh", "common.cuh")
+ATTN_TRAFFIC = {"70f60df556869cd5": 314053888}
 
 DEFAULT_WORKLOAD = "serve32"
 # the target model width behind each configuration's LM head (for the fused
@@ -69,10 +70,14 @@ def workload_text(w, layers, phys) -> str:
 
 
 def attn_source_digest() -> str:
+    """sha256 prefix of the sources the tree-attention launch is built from:
+    the kernel, its launch and schedule, and the PTX helpers it inlines."""
     import hashlib
-    src = os.path.join(ROOT, "paper_2608_00531_gb300", "csrc", "k_attn_tc.cu")
-    with open(src, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for name in ATTN_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_00531_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def peaks():
