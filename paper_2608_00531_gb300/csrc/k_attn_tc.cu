@@ -17,7 +17,7 @@
 //   warps 0-3 / 4-7   softmax of M tile 0 / 1: thread t owns row t = TMEM lane t
 //                     and writes its bf16 probabilities back into TMEM
 //   warp 8            TMA producer: Q rows (4-D box: d x group head x node),
-//                     64-key K and V tiles into 4-stage rings (128-byte
+//                     64-key K and V tiles into 5-stage rings (128-byte
 //                     swizzle), page ids prefetched, boxes issued from
 //                     several lanes.  A tile from a paged cache is
 //                     [8-key group][d half][8 keys][64 d] for K and V alike:
@@ -64,7 +64,7 @@ using namespace tc;
 constexpr int BM = kAttnRowsCta;  // 128 rows per M tile
 constexpr int BN = kAttnKeys;     // 64 keys per tile
 constexpr int D = kAttnD;         // 128
-constexpr int NS = 4;             // K and V ring stages
+constexpr int NS = 5;             // K and V ring stages
 constexpr int kThreads = 384;     // 12 warps
 constexpr uint32_t kTmemCols = 512;
 
@@ -776,21 +776,6 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
           const bool need = m_new > m_run + 8.0f;
           const float m_use = need ? m_new : m_run;
           const float nbase = m_use == -INFINITY ? 0.f : -m_use;
-          // exponent arguments and row sums two at a time (packed f32x2)
-          uint32_t pk[32];
-          const uint64_t c2 = f2_pack(c, c), nb2 = f2_pack(nbase, nbase);
-          uint64_t sm2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            float a0, a1;
-            f2_unpack(f2_fma(f2_pack(x[2 * i], x[2 * i + 1]), c2, nb2), a0, a1);
-            const float p0 = ex2(a0), p1 = ex2(a1);
-            sm2[i & 1] = f2_add(sm2[i & 1], f2_pack(p0, p1));
-            pk[i] = pack_bf16(p0, p1);
-          }
-          float sm[4];
-          f2_unpack(sm2[0], sm[0], sm[1]);
-          f2_unpack(sm2[1], sm[2], sm[3]);
           // P(t) goes into buffer t & 1 once PV(t - 2), which read it last, is
           // done (each buffer has its own done barrier: PV(t) completes phase
           // t >> 1 of barrier t & 1, and PV(t) cannot start before P(t) is
@@ -799,7 +784,28 @@ tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_const
             if (!wait_warp(bar(B_PVDONE + 2 * m + pbuf), ((tcur >> 1) & 1u) ^ 1u, abort_flag, A.err)) { ok = false; break; }
             tc_fence_after();
           }
-          tmem_st32(tl + kColP + m * 64 + pbuf * 32, pk);
+          // exponent arguments and row sums two at a time (packed f32x2); each
+          // half of P goes to TMEM as soon as it is computed, so that the first
+          // half's store runs under the second half's exponentials
+          uint32_t pk[32];
+          const uint64_t c2 = f2_pack(c, c), nb2 = f2_pack(nbase, nbase);
+          uint64_t sm2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
+          auto exp_pair = [&](int i) {
+            float a0, a1;
+            f2_unpack(f2_fma(f2_pack(x[2 * i], x[2 * i + 1]), c2, nb2), a0, a1);
+            const float p0 = ex2(a0), p1 = ex2(a1);
+            sm2[i & 1] = f2_add(sm2[i & 1], f2_pack(p0, p1));
+            pk[i] = pack_bf16(p0, p1);
+          };
+#pragma unroll
+          for (int i = 0; i < 16; ++i) exp_pair(i);
+          tmem_st16(tl + kColP + m * 64 + pbuf * 32, pk);
+#pragma unroll
+          for (int i = 16; i < 32; ++i) exp_pair(i);
+          tmem_st16(tl + kColP + m * 64 + pbuf * 32 + 16, pk + 16);
+          float sm[4];
+          f2_unpack(sm2[0], sm[0], sm[1]);
+          f2_unpack(sm2[1], sm[2], sm[3]);
           // O_m is rescaled only once PV(t - 1) is done
           if (jj > 0 && __any_sync(0xffffffffu, need)) {
             const uint32_t tp = tcur - 1;
