@@ -41,6 +41,10 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+# the CPU baseline is the oracle on one host thread: numpy's BLAS pool is
+# sized from these before numpy loads
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
@@ -596,7 +600,6 @@ def main():
         run_reference(args)
         return
 
-    os.environ.setdefault("OMP_NUM_THREADS", "1")
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     if world > 1:
