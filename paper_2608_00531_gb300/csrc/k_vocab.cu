@@ -535,6 +535,10 @@ vocab_ring_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
 // logit wants many resident warps): every thread streams 16-byte vectors with
 // non-allocating loads, the next vectors loaded while the current ones are
 // consumed.  grid (S, rows) with cluster (S, 1, 1).
+// Vectors per lane per step of the register-streaming scan: three 16-byte
+// loads in flight per lane (70 registers, still one wave of the grid).
+constexpr int kUnrollS = 3;
+
 template <int KT, bool LSE, bool TARGET>
 __global__ void __launch_bounds__(kThreads)
 vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int n_max,
@@ -586,29 +590,29 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
   //    term and the rescale is rare and uniform.
   const int lane = tid & 31;
   const int wb0 = vb + (tid & ~31);
-  uint4 r[kUnroll];
+  uint4 r[kUnrollS];
 #pragma unroll
-  for (int u = 0; u < kUnroll; ++u) {
+  for (int u = 0; u < kUnrollS; ++u) {
     const int vi = wb0 + lane + u * kThreads;
     if (vi < ve) r[u] = ld_stream(vp + vi);
   }
   float thr = warp_kth(tk);
   float mbw = -INFINITY;
   uint64_t sacc = f2_pack(0.f, 0.f);  // two lane sums, as one f32x2 pair
-  // one step: kUnroll vectors per lane; FULL when every lane's vectors are in
+  // one step: kUnrollS vectors per lane; FULL when every lane's vectors are in
   // range (all but a warp's last step), so that no per-vector check is needed
   auto step = [&](int wb, auto full_tag) {
     constexpr bool FULL = decltype(full_tag)::value;
-    uint4 nx[kUnroll];
+    uint4 nx[kUnrollS];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int vi = wb + lane + (kUnroll + u) * kThreads;
+    for (int u = 0; u < kUnrollS; ++u) {
+      const int vi = wb + lane + (kUnrollS + u) * kThreads;
       if (vi < ve) nx[u] = ld_stream(vp + vi);
     }
-    uint64_t xp[kUnroll][4];  // (lo, hi) logit pairs of each 32-bit word
-    float gmv[kUnroll];
+    uint64_t xp[kUnrollS][4];  // (lo, hi) logit pairs of each 32-bit word
+    float gmv[kUnrollS];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
+    for (int u = 0; u < kUnrollS; ++u) {
       const uint32_t w[4] = {r[u].x, r[u].y, r[u].z, r[u].w};
       float lo[4], hi[4];
 #pragma unroll
@@ -623,7 +627,7 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     if constexpr (LSE) {
       float gl = gmv[0];
 #pragma unroll
-      for (int u = 1; u < kUnroll; ++u) gl = fmaxf(gl, gmv[u]);
+      for (int u = 1; u < kUnrollS; ++u) gl = fmaxf(gl, gmv[u]);
       if (__any_sync(0xffffffffu, gl * kLog2e > mbw + 8.f)) {
         const float nb = warp_max(gl) * kLog2e;
         if (mbw != -INFINITY) {
@@ -635,7 +639,7 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       if (mbw != -INFINITY) {
         const uint64_t l2 = f2_pack(kLog2e, kLog2e), nb2 = f2_pack(-mbw, -mbw);
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
+        for (int u = 0; u < kUnrollS; ++u) {
           if (FULL || wb + lane + u * kThreads < ve) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -654,7 +658,7 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       // that a warp does not start by inserting every logit it sees
       float gl = gmv[0];
 #pragma unroll
-      for (int u = 1; u < kUnroll; ++u) gl = fmaxf(gl, gmv[u]);
+      for (int u = 1; u < kUnrollS; ++u) gl = fmaxf(gl, gmv[u]);
 #pragma unroll
       for (int k = 0; k < KT; ++k) {
         const float mk = warp_max(gl);
@@ -664,10 +668,10 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
     }
     bool cand = false;
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) cand |= (FULL || wb + lane + u * kThreads < ve) && gmv[u] >= thr;
+    for (int u = 0; u < kUnrollS; ++u) cand |= (FULL || wb + lane + u * kThreads < ve) && gmv[u] >= thr;
     if (__any_sync(0xffffffffu, cand)) {
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
+      for (int u = 0; u < kUnrollS; ++u) {
         if ((FULL || wb + lane + u * kThreads < ve) && gmv[u] >= thr) {
           const int idx = a0 + ((wb + lane + u * kThreads) << 3);
 #pragma unroll
@@ -682,12 +686,12 @@ vocab_scan_kernel(const uint16_t* __restrict__ logits, int vocab, int k_out, int
       thr = warp_kth(tk);
     }
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) r[u] = nx[u];
+    for (int u = 0; u < kUnrollS; ++u) r[u] = nx[u];
   };
   int wb = wb0;
-  for (; wb + 31 + (kUnroll - 1) * kThreads < ve; wb += kUnroll * kThreads)
+  for (; wb + 31 + (kUnrollS - 1) * kThreads < ve; wb += kUnrollS * kThreads)
     step(wb, std::integral_constant<bool, true>());
-  for (; wb < ve; wb += kUnroll * kThreads) step(wb, std::integral_constant<bool, false>());
+  for (; wb < ve; wb += kUnrollS * kThreads) step(wb, std::integral_constant<bool, false>());
   float sa, sb2;
   f2_unpack(sacc, sa, sb2);
   const float s0 = sa, s1 = sb2;
