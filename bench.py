@@ -415,43 +415,48 @@ def stage_roofs(alg, pk, w, Ly):
 
 
 def timed_steps(st, xs, kcs, vcs, steps, stream, world, dev, events=True):
-    """`steps` steps cycling over the input sets, with an event pair around
-    each stage group; returns the total device ms and the per-stage ms."""
+    """`steps` steps cycling over the input sets; returns the total device ms
+    and, with `events`, the per-stage ms from an event pair around each stage
+    group (an event between two launches keeps the second from starting its
+    set-up under the first, so the step's own time is taken without them)."""
     from paper_2608_00531_gb300 import cure
     P = len(xs)
     Ly = st.layers
     names = ("scan", "tree", "attn", "accept", "resync")
     ev = {k_: [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)] for k_ in names}
 
+    def mark(k_, s, i):
+        if events:
+            ev[k_][s][i].record(stream)
+
     def one(s):
         x = xs[s % P]
-        e = ev["scan"][s]
-        e[0].record(stream)
+        mark("scan", s, 0)
         cure.cure_score_draft(x.draft_logits, st.k, out=st.score)
-        e[1].record(stream)
-        ev["tree"][s][0].record(stream)
+        mark("scan", s, 1)
+        mark("tree", s, 0)
         tree = cure.cure_build_tree(st.score[0], st.score[2], x.root_tok, x.cache_len, st.tau, st.R,
                                     st.branches, st.depth, x.redraft, st.max_ufp, out=st.tree)
-        ev["tree"][s][1].record(stream)
+        mark("tree", s, 1)
         # one event pair around the step's attention launches (events between
         # the launches would stop each from starting its set-up under the
         # previous one, which it does as a programmatic dependent launch)
-        ev["attn"][s][0].record(stream)
+        mark("attn", s, 0)
         for l in range(Ly):
             p_ = st.layer_map[l]
             cure.cure_tree_attn(x.q[l], x.tree_k[l], x.tree_v[l], kcs[p_], vcs[p_], st.kv, x.cache_len,
                                 tree["n_nodes"], tree["anc"], st.scale, out=st.attn_out[l],
                                 workspace=st.workspace)
-        ev["attn"][s][1].record(stream)
-        ev["accept"][s][0].record(stream)
+        mark("attn", s, 1)
+        mark("accept", s, 0)
         acc = cure.cure_accept(tree, st.K, target_logits=x.target_logits, targ=st.targ, out=st.acc)
-        ev["accept"][s][1].record(stream)
-        ev["resync"][s][0].record(stream)
+        mark("accept", s, 1)
+        mark("resync", s, 0)
         kl = [kcs[st.layer_map[l]] for l in range(Ly)]
         vl = [vcs[st.layer_map[l]] for l in range(Ly)]
         cure.cure_resync_kv(kl, vl, st.kv, x.tree_k, x.tree_v, acc, x.cache_len, st.K,
                             cache_len_out=st.cache_len_out, out=st.rs)
-        ev["resync"][s][1].record(stream)
+        mark("resync", s, 1)
 
     if world > 1:
         import torch.distributed as dist
@@ -465,8 +470,10 @@ def timed_steps(st, xs, kcs, vcs, steps, stream, world, dev, events=True):
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1), world, dev)
-    per = {k_: float(np.mean([ev[k_][s][0].elapsed_time(ev[k_][s][1]) for s in range(steps)])) for k_ in names}
-    per["attn"] /= Ly
+    per = None
+    if events:
+        per = {k_: float(np.mean([ev[k_][s][0].elapsed_time(ev[k_][s][1]) for s in range(steps)])) for k_ in names}
+        per["attn"] /= Ly
     return ms, per
 
 
@@ -511,7 +518,8 @@ def sweep_points(wl, dev, steps, warmup, world, rank):
                         while e < K and tok[b, e + 1] == targ[b, e]:
                             e += 1
                         prefix_ok &= bool(a[b] == e)
-            ms, per = timed_steps(st, xs, p["kcs"], p["vcs"], steps, stream, world, dev)
+            ms, _ = timed_steps(st, xs, p["kcs"], p["vcs"], steps, stream, world, dev, events=False)
+            _, per = timed_steps(st, xs, p["kcs"], p["vcs"], steps, stream, world, dev)
             algs = [algorithmic(p, th) for th in p["trees"]]
             out.append({"budget": R, "tau": tau, "steps_per_s": round(job_steps_per_s(ms, steps, world), 2),
                         "ms_per_step": round(ms / steps, 4),
@@ -626,13 +634,17 @@ def main():
     clk.start()
     with quiet_host():
         clk.mark_start()
-        ms, per = timed_steps(st, xs, kcs, vcs, args.steps, stream, world, dev)
+        ms, _ = timed_steps(st, xs, kcs, vcs, args.steps, stream, world, dev, events=False)
         clk.mark_stop()
     clocks = clk.stop()
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
     assert cure.cure_device_error() == 0
+    # the per-stage times from a second pass of the same steps, with an event
+    # pair around each stage group
+    with quiet_host():
+        _, per = timed_steps(st, xs, kcs, vcs, args.steps, stream, world, dev)
     attn_avg, scan_avg, acc_avg, rs_ms = per["attn"], per["scan"], per["accept"], per["resync"]
     rs_b = float(np.mean([resync_bytes(acc_lens[i], Ly, w.heads_kv) for i in sel]))
 
