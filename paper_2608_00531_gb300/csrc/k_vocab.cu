@@ -39,7 +39,7 @@ namespace {
 constexpr int kThreads = 128;              // consumer threads (4 warps)
 constexpr int kWarps = kThreads / 32;
 constexpr int kCtaThreads = kThreads + 32; // plus one producer warp
-constexpr int kUnroll = 2;                 // vectors per lane per step
+constexpr int kUnroll = 2;                 // vectors per consumer lane per step (ring-fed scan)
 constexpr int kChunkVec = 512;             // 16-byte vectors per ring stage (8 KiB)
 constexpr int kStages = 3;
 constexpr float kLog2e = 1.4426950408889634f;
