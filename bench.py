@@ -963,8 +963,8 @@ def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
         fields += ("redraft",)
     host = {k_: getattr(x, k_).cpu().pin_memory() for k_ in fields}
     outs = torch.empty(4, st.B, st.K + 2, dtype=torch.int32).pin_memory()
-    h2d = sum(v.numel() * v.element_size() for v in host.values())
-    d2h = outs.numel() * outs.element_size()
+    d2h = outs.numel() * outs.element_size() + (st.B * 4 if x.target_logits.numel() * 2 >= st.NODE_ROWS_MIN_BYTES else 0)  # results; node counts read mid-step
+    h2d_steps = []
     stream = torch.cuda.current_stream()
     xh = StepInputs(host["draft_logits"], host["root_tok"], host["cache_len"], host.get("redraft"), host["q"],
                     host["tree_k"], host["tree_v"], host["target_logits"])
@@ -973,6 +973,7 @@ def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
         # the public step with host inputs: it streams them in on a copy
         # stream, each stage waiting for its own inputs
         r = st.run_from_host(xh, kcs, vcs)
+        h2d_steps.append(st.last_h2d_bytes)
         outs[0, :, 0].copy_(r["acc"]["accept_len"], non_blocking=True)
         outs[1].copy_(r["acc"]["out_tokens"], non_blocking=True)
         outs[2].copy_(r["resync"]["replay_tokens"], non_blocking=True)
@@ -993,6 +994,7 @@ def run_e2e(wl, st, kcs, vcs, dev, steps, world=1):
     b.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(a.elapsed_time(b), world, dev) / steps
+    h2d = float(np.mean(h2d_steps[-steps:]))
     return {"value": round(job_steps_per_s(ms * steps, steps, world), 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 4), "steps": steps}
 
