@@ -504,6 +504,22 @@ def test_tree_attn_full_serve_layer_sampled(cure):
     _cmp_attn(got, ref, t, seqs)
 
 
+def test_tree_attn_maximum_batch(cure):
+    """256 sequences, the most one call takes: the per-sequence prefix sums
+    span eight warp-wide passes and the schedule holds 1024 units over the
+    CTAs; short ragged caches (0 to 300 keys, paged) and trees of up to 9
+    nodes, every sequence checked against the oracle."""
+    B, K, budget = 256, 4, 4
+    rng = np.random.default_rng(256)
+    lens = rng.integers(0, 301, size=B)
+    lens[:4] = [0, 1, 64, 300]
+    t, q, tk, tv, kc, vc, L, table, npages = _attn_case(B, K, budget, 32, 8, lens, True, 1.0, 1.0, seed=256)
+    got = _run_attn(cure, t, q, tk, tv, kc, vc, L, table, npages, 8)
+    ref = oracle.tree_attn(_f64(q), _f64(tk), _f64(tv), _f64(kc), _f64(vc), L, t["n_nodes"], t["anc"],
+                           1.0 / math.sqrt(128), table, 16)
+    _cmp_attn(got, ref, t)
+
+
 @pytest.mark.parametrize("name,budget", [("single8b", None), ("long64", None), ("sweep16", 64)])
 def test_tree_attn_config_layer_sampled(cure, name, budget):
     """One layer at the other configurations' full shapes, contiguous caches:
@@ -1030,12 +1046,19 @@ def test_full_step_serve_shape(cure):
     xh = StepInputs(d.logits.pin_memory(), torch.from_numpy(d.root_tok).pin_memory(),
                     torch.from_numpy(L).pin_memory(), None, q.pin_memory(), tk.pin_memory(), tv.pin_memory(),
                     tl.pin_memory())
-    for _ in range(2):
+    # first with the target logits copied by node rows, then whole (a
+    # threshold above their size): the same results, fewer bytes the first way
+    h2d = []
+    for thr in (RepairVerifyStep.NODE_ROWS_MIN_BYTES, 1 << 62):
+        st.NODE_ROWS_MIN_BYTES = thr
         r2 = st.run_from_host(xh, kcs, vcs)
         torch.cuda.synchronize()
         assert cure.cure_device_error() == 0
+        h2d.append(st.last_h2d_bytes)
         for (grp, key), v in ints.items():
             assert torch.equal(r2[grp][key], v), (grp, key)
         for b in range(B):
             nb = int(t["n_nodes"][b])
             assert float((r2["attn"][:, b, :nb].float() - attn[:, b, :nb]).abs().max()) <= 1e-2, b
+    row_bytes = w.vocab * 2
+    assert h2d[1] - h2d[0] == int((N - t["n_nodes"]).sum()) * row_bytes
