@@ -70,10 +70,11 @@ def _check(got, h64, w, d, want=None):
 
 
 @pytest.mark.parametrize("rows,d,V", [(1, 64, 256), (37, 128, 1000), (130, 256, 4099), (300, 192, 20000),
-                                      (129, 4096, 3001)])
+                                      (129, 4096, 3001), (64, 8192, 20011)])
 def test_lm_head_argmax_small_shapes(cure, rows, d, V):
     """Ragged rows (M tails), vocabularies ending inside an N tile, several
-    K slices; unplanted rows, so the argmax is decided by noise."""
+    K slices (up to d_model 8192, the 70B-class width: 128 of them); unplanted
+    rows, so the argmax is decided by noise."""
     rng = np.random.default_rng(rows * 7 + V)
     h = W.to_bf16(rng.standard_normal((rows, d)).astype(np.float32))
     w = W.to_bf16((rng.standard_normal((V, d)) / np.sqrt(d)).astype(np.float32))
